@@ -1,0 +1,69 @@
+"""Seeded synthetic inputs shared by the tests, the smoke check and the benchmark.
+
+This module holds no attention or expansion arithmetic: it only draws random
+tensors with a CPU ``torch.Generator`` so the CUDA path and the CPU oracle can
+be fed identical bytes.  The shapes mirror the paper's workloads (Qwen3-8B-class
+dense attention: Hq=32, Hkv=8, Dh=128; large-MoE-class: Hq=64, Hkv=8, Dh=128;
+expansion factors n in {1, 2, 4, 8}); the paper's data and weights are not
+available, so N(0, 1) activations and N(0, 0.02) embedding tables stand in.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+WITHIN, CROSS, LOCAL = 0, 1, 2
+
+
+@dataclass(frozen=True)
+class AttnShape:
+    B: int
+    L: int        # tokens per sequence (before expansion)
+    n: int        # expansion factor (streams per token)
+    Hq: int
+    Hkv: int
+    Dh: int
+
+    @property
+    def nL(self) -> int:
+        return self.n * self.L
+
+
+# Named workloads (tokens L before expansion; the kernels see n*L positions).
+SHAPES = {
+    "tiny": AttnShape(1, 64, 2, 4, 4, 64),
+    "qwen3_8b_n4": AttnShape(1, 4096, 4, 32, 8, 128),
+    "moe_large_n4": AttnShape(1, 8192, 4, 64, 8, 128),
+}
+
+
+def _randn(shape, seed: int, std: float = 1.0) -> torch.Tensor:
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed)
+    x = torch.randn(shape, generator=g, dtype=torch.float32)
+    if std != 1.0:
+        x.mul_(std)
+    return x.to(torch.bfloat16)
+
+
+def attn_inputs(s: AttnShape, seed: int = 0, with_grad: bool = True):
+    """Q, K, V (and dO) in bf16, N(0, 1), layouts [B][nL][H][Dh].
+
+    Seeds: seed+0 -> Q, seed+1 -> K, seed+2 -> V, seed+3 -> dO."""
+    q = _randn((s.B, s.nL, s.Hq, s.Dh), seed)
+    k = _randn((s.B, s.nL, s.Hkv, s.Dh), seed + 1)
+    v = _randn((s.B, s.nL, s.Hkv, s.Dh), seed + 2)
+    if not with_grad:
+        return q, k, v
+    do = _randn((s.B, s.nL, s.Hq, s.Dh), seed + 3)
+    return q, k, v, do
+
+
+def embed_inputs(B: int, L: int, n: int, V: int, D: int, seed: int = 0):
+    """n embedding tables bf16 [n][V][D] ~ N(0, 0.02) and token ids int32 [B][L] ~ U[0, V)."""
+    tables = _randn((n, V, D), seed, std=0.02)
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed + 1000)
+    ids = torch.randint(0, V, (B, L), generator=g, dtype=torch.int64).to(torch.int32)
+    return tables, ids
