@@ -1,0 +1,470 @@
+#!/usr/bin/env python
+"""Benchmark of the Stream-Factorized Attention hot path on GB300.
+
+One step = one pass of the hot path over one synthetic batch of the
+Qwen3-8B-class layer (B=1, L=4096 tokens, n=4 -> 16384 positions, Hq=32, Hkv=8,
+Dh=128, bf16, intra-stream / WITHIN mask):
+  expansion gather (4 tables of 151936 x 4096)  -> sfa_fwd -> sfa_bwd_prep
+  -> sfa_bwd_main -> sfa_bwd_finalize.
+Metric: attention FLOPs over visible pairs only (forward 4*Dh, backward 10*Dh per
+pair and query head) per second of the whole step, in TFLOP/s.
+
+The same JSON line also carries: the dominant kernel's roofline, the end-to-end
+number through the C ABI with host buffers, the CPU oracle baseline, the CROSS
+(full cross-stream) layer of the same shape and the expansion-factor sweep.
+
+--impl reference times the fp64 CPU oracle on a bounded sample of the same
+workload (the paper publishes no implementation to run).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, SHAPES, WITHIN, attn_inputs  # noqa: E402
+
+METRIC = "SFA fwd+bwd TFLOP/s (visible pairs) at n=4, % of bf16 peak; scaling vs n"
+WORKLOAD = "qwen3_8b_n4"
+GATHER_V, GATHER_D = 151936, 4096
+FWD_FLOP, BWD_FLOP = 4, 10  # per visible pair, per query head, times Dh
+MODE_NAME = {WITHIN: "WITHIN", CROSS: "CROSS", LOCAL: "LOCAL"}
+
+
+# ---------------------------------------------------------------- FLOP model
+def visible_pairs(s: AttnShape, mode: int, window: int = 0) -> int:
+    """Visible (query, key) pairs per (batch, head): WITHIN n*L(L+1)/2 (Eq. 4),
+    CROSS nL(nL+1)/2 (Fig. 2a), LOCAL sum_p min(p+1, w) (Fig. 2b)."""
+    if mode == WITHIN:
+        return s.n * s.L * (s.L + 1) // 2
+    if mode == CROSS:
+        return s.nL * (s.nL + 1) // 2
+    w = min(window, s.nL)
+    return w * (w + 1) // 2 + (s.nL - w) * w
+
+
+def attn_flops(s: AttnShape, mode: int, per_pair: int, window: int = 0) -> float:
+    return float(per_pair) * s.Dh * visible_pairs(s, mode, window) * s.Hq * s.B
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"bf16": p["bf16_tflops"], "bf16_sustained": p["bf16_tflops_sustained"],
+                "hbm": p["hbm_gbs"], "src": "measured"}
+    except Exception:
+        return {"bf16": 1900.0, "bf16_sustained": 1700.0, "hbm": 6800.0, "src": "fallback"}
+
+
+# ---------------------------------------------------------------- distributed
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def reduce_max(x: float, ws: int) -> float:
+    """Max of a per-rank number over all ranks (the job's time is its slowest rank)."""
+    if ws <= 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: float, seconds_per_rank: float, ws: int) -> tuple[float, float]:
+    """Weak scaling: every rank processes its own batch; value = all ranks' units / slowest time."""
+    t = reduce_max(seconds_per_rank, ws)
+    return units_per_rank * ws / t, t
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"hdsfa_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for ln in f:
+                parts = [p.strip() for p in ln.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, val in zip(names, parts[5:9]):
+                    if val.lower() == "active":
+                        reasons.add(nm)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------- the step
+class HotPath:
+    """Device buffers and the five launches of one step."""
+
+    def __init__(self, s: AttnShape, mode: int, dev, with_gather: bool = True, seed: int = 1):
+        from paper_2607_08186_gb300 import binding
+        self.b = binding
+        self.s, self.mode, self.dev = s, mode, dev
+        q, k, v, do = attn_inputs(s, seed=seed)
+        self.host_in = [t.pin_memory() for t in (q, k, v, do)]
+        self.q, self.k, self.v, self.do = (t.to(dev, non_blocking=False) for t in self.host_in)
+        self.o = torch.empty_like(self.q)
+        self.lse = torch.empty(s.B, s.Hq, s.nL, dtype=torch.float32, device=dev)
+        self.dq, self.dk, self.dv = torch.empty_like(self.q), torch.empty_like(self.k), torch.empty_like(self.v)
+        self.ws = torch.empty(binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),
+                              dtype=torch.uint8, device=dev)
+        self.with_gather = with_gather
+        if with_gather:
+            g = torch.Generator(device=dev)
+            g.manual_seed(seed + 100)
+            # n embedding tables ~ N(0, 0.02), Qwen3-8B-sized (V x D = 0.62B per table)
+            self.tables = (torch.randn(s.n, GATHER_V, GATHER_D, generator=g, device=dev,
+                                       dtype=torch.float32) * 0.02).to(torch.bfloat16)
+            gi = torch.Generator().manual_seed(seed + 200)
+            self.host_ids = torch.randint(0, GATHER_V, (s.B, s.L), generator=gi,
+                                          dtype=torch.int64).to(torch.int32).pin_memory()
+            self.ids = self.host_ids.to(dev)
+            self.x = torch.empty(s.B, s.nL, GATHER_D, dtype=torch.bfloat16, device=dev)
+        self.host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                         for t in (self.o, self.lse, self.dq, self.dk, self.dv)]
+        self.launches_per_step = 4 + (1 if with_gather else 0)
+
+    def step(self, ev=None):
+        b, s = self.b, self.s
+        if self.with_gather:
+            b.hd_expand_embed(self.tables, self.ids, self.x)
+        if ev is not None:
+            ev[0].record()
+        b.sfa_fwd(self.q, self.k, self.v, self.o, self.lse, s.n, self.mode)
+        if ev is not None:
+            ev[1].record()
+        b.sfa_bwd_prep(self.o, self.do, s.n, self.mode, self.ws, s.Hkv)
+        if ev is not None:
+            ev[2].record()
+        b.sfa_bwd_main(self.q, self.k, self.v, self.lse, self.do, self.dk, self.dv, s.n, self.mode, self.ws)
+        if ev is not None:
+            ev[3].record()
+        b.sfa_bwd_finalize(self.dq, s.n, self.mode, self.ws, s.Hkv)
+
+    def step_e2e(self):
+        """Host -> device inputs, the step, device -> host results (pinned buffers)."""
+        for dst, src in zip((self.q, self.k, self.v, self.do), self.host_in):
+            dst.copy_(src, non_blocking=True)
+        if self.with_gather:
+            self.ids.copy_(self.host_ids, non_blocking=True)
+        self.step()
+        for dst, src in zip(self.host_out, (self.o, self.lse, self.dq, self.dk, self.dv)):
+            dst.copy_(src, non_blocking=True)
+
+    def io_bytes(self):
+        h2d = sum(t.numel() * t.element_size() for t in self.host_in)
+        if self.with_gather:
+            h2d += self.host_ids.numel() * 4
+        d2h = sum(t.numel() * t.element_size() for t in self.host_out)
+        return h2d, d2h
+
+
+def time_loop(fn, steps, warmup, ws):
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    barrier(ws)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        fn()
+    t1.record()
+    torch.cuda.synchronize()
+    barrier(ws)
+    return t0.elapsed_time(t1) / 1e3 / steps
+
+
+def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2):
+    """fwd, bwd-main and fwd+bwd times of one layer (no gather), seconds."""
+    hp = HotPath(s, mode, dev, with_gather=False, seed=7)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(iters)]
+    for _ in range(warmup):
+        hp.step()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for i in range(iters):
+        hp.step(evs[i])
+    t1.record()
+    torch.cuda.synchronize()
+    total = t0.elapsed_time(t1) / 1e3 / iters
+    fwd = statistics.median(e[0].elapsed_time(e[1]) for e in evs) / 1e3
+    bwd = statistics.median(e[2].elapsed_time(e[3]) for e in evs) / 1e3
+    del hp
+    torch.cuda.empty_cache()
+    return {"fwd_s": fwd, "bwd_main_s": bwd, "step_s": total}
+
+
+# ---------------------------------------------------------------- ncu traffic record
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_08186_gb300", "csrc")
+    for fn in sorted(os.listdir(csrc)):
+        if fn.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, fn), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_record(kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it was
+    taken on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    m = re.search(rf"^\| {re.escape(kernel)} \| ([0-9a-f]+) \| ([0-9.e+]+) \|", txt, flags=re.M)
+    if not m or m.group(1) != kernel_source_hash():
+        return None
+    return float(m.group(2))
+
+
+# ---------------------------------------------------------------- CPU oracle baseline
+def oracle_prefix_sample(L_prefix: int, mode: int):
+    """fp64 oracle fwd + bwd of the benchmark layer restricted to its first
+    L_prefix tokens (all heads).  Returns (seconds, visible-pair FLOPs)."""
+    import oracle
+    full = SHAPES[WORKLOAD]
+    sp = AttnShape(full.B, L_prefix, full.n, full.Hq, full.Hkv, full.Dh)
+    q, k, v, do = attn_inputs(sp, seed=1)
+    t = time.perf_counter()
+    oracle.sfa_fwd(q, k, v, sp.n, mode)
+    oracle.sfa_bwd(q, k, v, do, sp.n, mode)
+    dt = time.perf_counter() - t
+    return dt, attn_flops(sp, mode, FWD_FLOP + BWD_FLOP), sp
+
+
+def cpu_baseline(target_s: float = 12.0, mode: int = WITHIN):
+    import oracle
+    oracle.build()
+    L0 = 64
+    t0, _, _ = oracle_prefix_sample(L0, mode)
+    Lp = int(L0 * math.sqrt(max(target_s, 0.5) / max(t0, 1e-3)))
+    Lp = max(L0, min(SHAPES[WORKLOAD].L, (Lp // 16) * 16))
+    dt, fl, sp = oracle_prefix_sample(Lp, mode)
+    return {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": (f"fp64 oracle fwd+bwd of the {MODE_NAME[mode]} layer on its first {Lp} tokens "
+                       f"({sp.nL} positions, Hq={sp.Hq}, Hkv={sp.Hkv}, Dh={sp.Dh}); "
+                       f"{dt:.1f} s for {fl:.3e} visible-pair FLOPs")}
+
+
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    budget = 150.0 / max(1, args.steps + args.warmup)
+    L0 = 64
+    t0, _, _ = oracle_prefix_sample(L0, WITHIN)
+    Lp = int(L0 * math.sqrt(max(budget, 0.3) / max(t0, 1e-3)))
+    Lp = max(16, min(SHAPES[WORKLOAD].L, (Lp // 16) * 16))
+    for _ in range(args.warmup):
+        oracle_prefix_sample(Lp, WITHIN)
+    times, fl, sp = [], 0.0, None
+    for _ in range(args.steps):
+        dt, fl, sp = oracle_prefix_sample(Lp, WITHIN)
+        times.append(dt)
+    mean = sum(times) / len(times)
+    val = fl / mean / 1e12
+    s = SHAPES[WORKLOAD]
+    sample = (f"each step: fp64 oracle fwd+bwd of the WITHIN layer on its first {Lp} tokens "
+              f"({sp.nL} positions, Hq={sp.Hq}, Hkv={sp.Hkv}, Dh={sp.Dh})")
+    print(json.dumps({
+        "metric": METRIC, "value": val, "unit": "TFLOP/s", "impl": "reference", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{WORKLOAD}_within: B={s.B} L={s.L} n={s.n} ({s.nL} positions) "
+                               f"Hq={s.Hq} Hkv={s.Hkv} Dh={s.Dh}, WITHIN mask", "sample": sample},
+        "cpu_baseline": {"value": val, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# ---------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-extras", action="store_true", help="skip CROSS layer, n sweep and CPU baseline")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    ws, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_08186_gb300 import build
+    if rank == 0 or ws == 1:
+        build.build()
+    barrier(ws)
+    s = SHAPES[WORKLOAD]
+    pk = peaks()
+    hp = HotPath(s, WITHIN, dev, with_gather=True, seed=1)
+    flops_step = attn_flops(s, WITHIN, FWD_FLOP + BWD_FLOP)
+
+    # device-resident timed region
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    it = iter(range(10 ** 9))
+    clocks = ClockSampler(local)
+
+    def timed():
+        i = next(it)
+        hp.step(evs[i - args.warmup] if i >= args.warmup else None)
+
+    for _ in range(args.warmup):
+        timed()
+    torch.cuda.synchronize()
+    barrier(ws)
+    clocks.start()
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        timed()
+    t1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(ws)
+    sec = t0.elapsed_time(t1) / 1e3 / args.steps
+    value, sec_max = job_throughput(flops_step, sec, ws)
+    fwd_s = statistics.mean(e[0].elapsed_time(e[1]) for e in evs) / 1e3
+    bwd_s = statistics.mean(e[2].elapsed_time(e[3]) for e in evs) / 1e3
+    bwd_flops = attn_flops(s, WITHIN, BWD_FLOP)
+    fwd_flops = attn_flops(s, WITHIN, FWD_FLOP)
+    dom = "sfa_bwd_main" if bwd_s >= fwd_s else "sfa_fwd"
+    dom_flops, dom_s = (bwd_flops, bwd_s) if dom == "sfa_bwd_main" else (fwd_flops, fwd_s)
+    achieved = dom_flops / dom_s / 1e12
+    tr = traffic_record(dom)
+
+    # end to end through the C ABI with host buffers
+    e2e_s = time_loop(hp.step_e2e, max(3, args.steps // 2), 2, ws)
+    e2e_val, _ = job_throughput(flops_step, e2e_s, ws)
+    h2d, d2h = hp.io_bytes()
+    launches = hp.launches_per_step * args.steps
+    del hp
+    torch.cuda.empty_cache()
+
+    out = {
+        "metric": METRIC, "value": value / 1e12, "unit": "TFLOP/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": sec_max * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": (f"{WORKLOAD}_within: B={s.B} L={s.L} n={s.n} ({s.nL} positions) "
+                                f"Hq={s.Hq} Hkv={s.Hkv} Dh={s.Dh}, WITHIN mask, fwd+bwd, plus the "
+                                f"expansion gather of {s.n} tables {GATHER_V}x{GATHER_D}"),
+                   "flops_per_step": flops_step, "flop_model": "fwd 4*Dh + bwd 10*Dh per visible pair per head",
+                   "l2": "inputs larger than L2 (Q 134 MB, dO 134 MB, K+V 67 MB, gather tables 5 GB)",
+                   "parallelism": f"replicas x{ws}"},
+        "pct_of_peak": 100.0 * value / 1e12 / pk["bf16"],
+        "roofline": {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": pk["bf16"],
+                     "unit": "TFLOP/s", "frac": achieved / pk["bf16"],
+                     "frac_of_sustained": achieved / pk["bf16_sustained"],
+                     "peak_source": f"{pk['src']} bf16 dense burst", "traffic": tr,
+                     "algorithmic_flops_per_launch": dom_flops, "avg_launch_ms": dom_s * 1e3},
+        "kernels_ms": {"sfa_fwd": fwd_s * 1e3, "sfa_bwd_main": bwd_s * 1e3},
+        "e2e": {"value": e2e_val / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3},
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if not args.no_extras and rank == 0 and ws == 1:
+        extras = {}
+        r = measure_layer(s, CROSS, dev)
+        fl = attn_flops(s, CROSS, FWD_FLOP + BWD_FLOP)
+        extras["cross_layer"] = {"workload": f"{WORKLOAD}_cross", "tflops": fl / r["step_s"] / 1e12,
+                                 "fwd_tflops": attn_flops(s, CROSS, FWD_FLOP) / r["fwd_s"] / 1e12,
+                                 "bwd_main_tflops": attn_flops(s, CROSS, BWD_FLOP) / r["bwd_main_s"] / 1e12,
+                                 "ms": r["step_s"] * 1e3}
+        sweep = []
+        for n in (1, 2, 4, 8):
+            sn = AttnShape(1, 4096, n, 32, 8, 128)
+            row = {"n": n}
+            for mode in (WITHIN, CROSS):
+                r = measure_layer(sn, mode, dev, iters=3, warmup=1)
+                fl = attn_flops(sn, mode, FWD_FLOP + BWD_FLOP)
+                row[MODE_NAME[mode]] = {"ms": r["step_s"] * 1e3, "tflops": fl / r["step_s"] / 1e12}
+            sweep.append(row)
+        base = sweep[0]["WITHIN"]["ms"]
+        for row in sweep:
+            row["WITHIN_cost_vs_n1"] = row["WITHIN"]["ms"] / base
+        extras["n_sweep"] = sweep
+        out["extras"] = extras
+        out["cpu_baseline"] = cpu_baseline()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

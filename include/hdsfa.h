@@ -1,0 +1,128 @@
+/*
+ * hdsfa.h -- C ABI of libhdsfa.so: GB300 (sm_103a) kernels for Hidden Decoding's
+ * multi-stream token expansion and Stream-Factorized Attention (SFA).
+ *
+ * Notation (0-indexed): a batch holds B sequences of L tokens; each token is
+ * expanded into n streams, giving nL positions.  Token t, stream s sits at
+ * position p = t*n + s (the paper's 1-indexed t = (i-1)n + k, Eq. 1).
+ *
+ * Conventions shared by every entry point
+ *   - Ownership: the caller allocates and owns every buffer (device memory).
+ *     The library never allocates, frees or synchronises; all work is enqueued
+ *     asynchronously on `stream` (0 = legacy default stream).
+ *   - Layout: dense row-major, no padding.  bf16 is IEEE bfloat16 (uint16 bits).
+ *       tables  [n][V][D]        ids [B][L] int32      expanded [B][nL][D]
+ *       q, o, dout, dq  [B][nL][Hq][Dh]      k, v, dk, dv  [B][nL][Hkv][Dh]
+ *       lse [B][Hq][nL] float32, natural-log log-sum-exp of each softmax row.
+ *   - Grouped K/V: query head h reads K/V head h / (Hq / Hkv).
+ *   - Host-side argument errors return before anything is enqueued.
+ *   - dev_status (nullable): a device int32 the kernels OR error bits into
+ *     (HD_DEVBIT_*); the caller zeroes it, synchronises, then reads it.
+ *     Kernels never trap.
+ *   - Pointers must be 16-byte aligned; D and Dh must make rows a multiple of
+ *     16 bytes.
+ */
+#ifndef HDSFA_H
+#define HDSFA_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  HD_OK = 0,
+  HD_ERR_INVALID_ARG = 1, /* null / misaligned pointer, non-positive size, Hq % Hkv != 0 */
+  HD_ERR_UNSUPPORTED = 2, /* valid but not implemented (e.g. Dh not in {64, 128}) */
+  HD_ERR_CUDA = 3,        /* a CUDA runtime/driver call or kernel launch failed */
+  HD_ERR_WORKSPACE = 4,   /* workspace null or smaller than sfa_bwd_workspace_bytes() */
+  HD_ERR_TIMEOUT = 5,     /* reserved: a bounded device wait expired (see HD_DEVBIT_TIMEOUT) */
+  HD_ERR_INDEX = 6        /* reserved: an index was out of range (see HD_DEVBIT_INDEX) */
+} hd_status_t;
+
+/* Bits the kernels OR into *dev_status. */
+#define HD_DEVBIT_INDEX 1   /* a token id outside [0, V): its n output rows were zeroed */
+#define HD_DEVBIT_TIMEOUT 2 /* a bounded pipeline wait expired; outputs are invalid */
+
+/* Attention mask of one SFA layer (Sec. 2.2, Eq. 4 and Fig. 2). */
+typedef enum {
+  SFA_WITHIN = 0, /* intra-stream: p' <= p and p' = p (mod n)                 (Eq. 4, Fig. 2c) */
+  SFA_CROSS = 1,  /* full cross-stream: standard causal mask over nL, p' <= p (Fig. 2a)        */
+  SFA_LOCAL = 2   /* local cross-stream: causal window, p - window < p' <= p  (Fig. 2b)        */
+} sfa_mode_t;
+
+/*
+ * hd_expand_embed -- multi-stream token expansion (Eq. 1, Sec. 2.1):
+ *   out[b][t*n + s][:] = tables[s][ids[b][t]][:]   for t < L, s < n.
+ * tables: bf16 [n][V][D] (read-only); ids: int32 [B][L]; out: bf16 [B][n*L][D].
+ * An id outside [0, V) writes zero rows and sets HD_DEVBIT_INDEX.
+ * Requires D % 8 == 0 (16-byte rows) and 16-byte aligned tables/out.
+ * Bit-exact copy; HBM-bound.
+ */
+hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L, int n,
+                            int V, int D, int32_t* dev_status, cudaStream_t stream);
+
+/*
+ * sfa_fwd -- SFA forward over the expanded sequence (Sec. 2.2; Eq. 3-4; Fig. 2):
+ *   O[b][p][h] = sum_{p' visible from p} softmax_p'(scale * q_p . k_p') v_p',
+ *   lse[b][h][p] = log sum_{p' visible} exp(scale * q_p . k_p').
+ * q: bf16 [B][nL][Hq][Dh]; k, v: bf16 [B][nL][Hkv][Dh]; o: bf16 like q (written);
+ * lse: float32 [B][Hq][nL] (written).  softmax_scale <= 0 selects 1/sqrt(Dh).
+ * window is used only by SFA_LOCAL (must be >= 1 there).  Dh in {64, 128}.
+ * Every position sees itself, so no softmax row is empty.
+ */
+hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
+                    int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode,
+                    int window, int32_t* dev_status, cudaStream_t stream);
+
+/* Bytes of device workspace sfa_bwd needs for these sizes (fp32 dQ accumulator
+ * [B][nL][Hq][Dh] plus fp32 row terms [B][Hq][nL]).  Returns 0 for invalid sizes. */
+size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode);
+
+/*
+ * sfa_bwd -- gradient of sfa_fwd (the paper trains with SFA but does not write
+ * the gradient; this is the derivative of the forward above):
+ *   P = exp(scale q k^T - lse) on visible pairs, dP = dO v^T,
+ *   dS = P * (dP - rowsum(dO * O)),
+ *   dq = scale dS k,  dk = scale sum_{h in group} dS^T q,  dv = sum_{h in group} P^T dO.
+ * Inputs q, k, v, o, dout (bf16) and lse (float32, as written by sfa_fwd).
+ * Outputs dq [B][nL][Hq][Dh], dk, dv [B][nL][Hkv][Dh] (bf16, overwritten).
+ * workspace: device buffer of at least sfa_bwd_workspace_bytes(...) bytes, 256-byte
+ * aligned; its contents on entry do not matter.
+ */
+hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                    const void* dout, void* dq, void* dk, void* dv, int B, int L, int n, int Hq,
+                    int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
+                    void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                    cudaStream_t stream);
+
+/*
+ * The three phases sfa_bwd runs, in order on one stream, exported so a caller
+ * can overlap or time them separately.  Same arguments and workspace as sfa_bwd.
+ *   sfa_bwd_prep     : delta[b][h][p] = sum_d dO*O (fp32) into the workspace and
+ *                      zero the workspace's fp32 dQ accumulator.
+ *   sfa_bwd_main     : recompute P, accumulate dQ (fp32, workspace) and write dk, dv.
+ *   sfa_bwd_finalize : dq = bf16(scale * accumulator).
+ * A later phase reads what the earlier one left in the workspace.
+ */
+hd_status_t sfa_bwd_prep(const void* o, const void* dout, int B, int L, int n, int Hq, int Hkv,
+                         int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
+                         cudaStream_t stream);
+hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const float* lse,
+                         const void* dout, void* dk, void* dv, int B, int L, int n, int Hq, int Hkv,
+                         int Dh, float softmax_scale, sfa_mode_t mode, int window, void* workspace,
+                         size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream);
+hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
+                             float softmax_scale, sfa_mode_t mode, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream);
+
+/* Human-readable name of a status code (static string). */
+const char* hd_status_string(hd_status_t status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HDSFA_H */

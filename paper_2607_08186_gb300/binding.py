@@ -1,0 +1,149 @@
+"""Thin ctypes binding over libhdsfa.so (C ABI in include/hdsfa.h).
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels of libhdsfa.so.  Functions keep the C names and take torch CUDA tensors
+(plain device memory); sizes are read from the tensor shapes.  There is no
+CPU fallback: if the library is missing or a call fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from .inputs import WITHIN, CROSS, LOCAL  # noqa: F401
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libhdsfa.so")
+_lock = threading.Lock()
+_lib = None
+
+HD_OK = 0
+HD_DEVBIT_INDEX = 1
+HD_DEVBIT_TIMEOUT = 2
+
+
+class HdError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {hd_status_string(code)} (code {code})")
+        self.code = code
+
+
+def lib():
+    """Load libhdsfa.so (built by ``build.build()``); raise if it is missing."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"libhdsfa.so is not built ({LIB_PATH}); run "
+                                   "paper_2607_08186_gb300.build.build() first")
+            L = ctypes.CDLL(LIB_PATH)
+            P, I, F, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+            L.hd_expand_embed.restype = I
+            L.hd_expand_embed.argtypes = [P, P, P, I, I, I, I, I, P, P]
+            L.sfa_fwd.restype = I
+            L.sfa_fwd.argtypes = [P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, P]
+            L.sfa_bwd_workspace_bytes.restype = Z
+            L.sfa_bwd_workspace_bytes.argtypes = [I, I, I, I, I, I, I]
+            L.sfa_bwd.restype = I
+            L.sfa_bwd.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
+            L.sfa_bwd_prep.restype = I
+            L.sfa_bwd_prep.argtypes = [P, P, I, I, I, I, I, I, I, P, Z, P]
+            L.sfa_bwd_main.restype = I
+            L.sfa_bwd_main.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
+            L.sfa_bwd_finalize.restype = I
+            L.sfa_bwd_finalize.argtypes = [P, I, I, I, I, I, I, F, I, P, Z, P]
+            L.hd_status_string.restype = ctypes.c_char_p
+            L.hd_status_string.argtypes = [I]
+            _lib = L
+    return _lib
+
+
+def hd_status_string(code: int) -> str:
+    return lib().hd_status_string(int(code)).decode()
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(code: int, where: str):
+    if code != HD_OK:
+        raise HdError(code, where)
+
+
+def hd_expand_embed(tables, ids, out, dev_status=None, stream=None):
+    """out[b][t*n+s] = tables[s][ids[b][t]]  (Eq. 1).  tables [n][V][D] bf16,
+    ids [B][L] int32, out [B][n*L][D] bf16."""
+    n, V, D = tables.shape
+    B, L = ids.shape
+    _check(lib().hd_expand_embed(_p(tables), _p(ids), _p(out), B, L, n, V, D, _p(dev_status),
+                                 _stream(stream)), "hd_expand_embed")
+    return out
+
+
+def _attn_dims(q, k, n):
+    B, nL, Hq, Dh = q.shape
+    if nL % n:
+        raise ValueError("q.shape[1] must be n * L")
+    return B, nL // n, Hq, k.shape[2], Dh
+
+
+def sfa_fwd(q, k, v, o, lse, n, mode, softmax_scale=0.0, window=0, dev_status=None, stream=None):
+    """SFA forward (Eq. 4 / Fig. 2 masks).  q,o [B][nL][Hq][Dh], k,v [B][nL][Hkv][Dh] bf16;
+    lse [B][Hq][nL] float32."""
+    B, L, Hq, Hkv, Dh = _attn_dims(q, k, n)
+    _check(lib().sfa_fwd(_p(q), _p(k), _p(v), _p(o), _p(lse), B, L, n, Hq, Hkv, Dh,
+                         float(softmax_scale), int(mode), int(window), _p(dev_status),
+                         _stream(stream)), "sfa_fwd")
+    return o, lse
+
+
+def sfa_bwd_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode) -> int:
+    return int(lib().sfa_bwd_workspace_bytes(B, L, n, Hq, Hkv, Dh, int(mode)))
+
+
+def sfa_bwd(q, k, v, o, lse, dout, dq, dk, dv, n, mode, workspace, softmax_scale=0.0, window=0,
+            dev_status=None, stream=None):
+    """SFA backward.  workspace: uint8 CUDA tensor of >= sfa_bwd_workspace_bytes bytes."""
+    B, L, Hq, Hkv, Dh = _attn_dims(q, k, n)
+    _check(lib().sfa_bwd(_p(q), _p(k), _p(v), _p(o), _p(lse), _p(dout), _p(dq), _p(dk), _p(dv),
+                         B, L, n, Hq, Hkv, Dh, float(softmax_scale), int(mode), int(window),
+                         _p(workspace), _wsb(workspace),
+                         _p(dev_status), _stream(stream)), "sfa_bwd")
+    return dq, dk, dv
+
+
+def _wsb(ws):
+    return ws.numel() * ws.element_size()
+
+
+def sfa_bwd_prep(o, dout, n, mode, workspace, Hkv, stream=None):
+    """Phase 1 of sfa_bwd: delta = rowsum(dO * O) and a zeroed dQ accumulator (workspace)."""
+    B, nL, Hq, Dh = o.shape
+    _check(lib().sfa_bwd_prep(_p(o), _p(dout), B, nL // n, n, Hq, Hkv, Dh, int(mode), _p(workspace),
+                              _wsb(workspace), _stream(stream)), "sfa_bwd_prep")
+
+
+def sfa_bwd_main(q, k, v, lse, dout, dk, dv, n, mode, workspace, softmax_scale=0.0, window=0,
+                 dev_status=None, stream=None):
+    """Phase 2 of sfa_bwd: dK, dV and the fp32 dQ accumulator."""
+    B, L, Hq, Hkv, Dh = _attn_dims(q, k, n)
+    _check(lib().sfa_bwd_main(_p(q), _p(k), _p(v), _p(lse), _p(dout), _p(dk), _p(dv), B, L, n, Hq,
+                              Hkv, Dh, float(softmax_scale), int(mode), int(window), _p(workspace),
+                              _wsb(workspace), _p(dev_status), _stream(stream)), "sfa_bwd_main")
+
+
+def sfa_bwd_finalize(dq, n, mode, workspace, Hkv, softmax_scale=0.0, stream=None):
+    """Phase 3 of sfa_bwd: dq = bf16(scale * accumulator)."""
+    B, nL, Hq, Dh = dq.shape
+    _check(lib().sfa_bwd_finalize(_p(dq), B, nL // n, n, Hq, Hkv, Dh, float(softmax_scale), int(mode),
+                                  _p(workspace), _wsb(workspace), _stream(stream)), "sfa_bwd_finalize")

@@ -1,0 +1,70 @@
+// Device helpers shared by the sm_103a kernels of libhdsfa.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/hdsfa.h"
+
+#define HD_DEVINLINE __device__ __forceinline__
+
+// One attention problem seen by a kernel: plain causal attention over a "virtual"
+// sequence of Lv rows whose row r lives at expanded position p = r*rs + s.
+//   WITHIN: one problem per stream s, Lv = L, rs = n   (Eq. 4: stream s sees only
+//           its own earlier positions, which are exactly every n-th row).
+//   CROSS : one problem, Lv = nL, rs = 1, s = 0       (Fig. 2a: causal over nL).
+//   LOCAL : as CROSS plus the window lower bound       (Fig. 2b).
+struct SfaGeom {
+  int B, nL, Hq, Hkv, n;
+  int Lv;       // rows of each virtual problem
+  int ns;       // problems per (b, head): n for WITHIN, 1 otherwise
+  int rs;       // expanded-position step between consecutive virtual rows
+  int window;   // > 0 only for LOCAL: key r' visible iff r - window < r' <= r
+};
+
+HD_DEVINLINE uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+HD_DEVINLINE void cp_async_16(uint32_t dst, const void* src, bool pred) {
+  int sz = pred ? 16 : 0;  // src-size 0 zero-fills the 16 destination bytes
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(sz));
+}
+HD_DEVINLINE void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+HD_DEVINLINE void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+
+HD_DEVINLINE void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+HD_DEVINLINE void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+
+// D(16x8 f32) += A(16x16 bf16, row) * B(16x8 bf16, col)
+HD_DEVINLINE void mma_bf16_16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+HD_DEVINLINE uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Element offset of (row, col) in a [rows][RL] bf16 tile whose 16-byte chunks are
+// XOR-swizzled by (row & 7), so 8 consecutive rows of one chunk hit 8 distinct
+// bank groups (conflict-free ldmatrix and cp.async).  RL must be >= 64.
+template <int RL>
+HD_DEVINLINE int swz(int row, int col) {
+  return row * RL + ((((col >> 3) ^ (row & 7))) << 3) + (col & 7);
+}
+
+HD_DEVINLINE void set_status(int32_t* st, int bit) {
+  if (st) atomicOr(st, bit);
+}

@@ -1,0 +1,190 @@
+// C ABI of libhdsfa.so (declared in include/hdsfa.h): host-side validation,
+// problem geometry and kernel dispatch.  No allocation, no synchronisation.
+#include <math.h>
+
+#include "common.cuh"
+
+namespace hdsfa {
+cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L,
+                                int n, int V, int D, int32_t* status, cudaStream_t stream);
+cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
+                               const SfaGeom& g, int Dh, float scale, cudaStream_t st);
+cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, float* delta_ws, float* dq_ws,
+                                const SfaGeom& g, int Dh, cudaStream_t st);
+cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const float* lse,
+                                    const void* dout, void* dk, void* dv, const float* delta_ws,
+                                    float* dq_ws, const SfaGeom& g, int Dh, float scale,
+                                    cudaStream_t st);
+cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
+                                    float scale, cudaStream_t st);
+}  // namespace hdsfa
+
+namespace {
+
+bool aligned16(const void* p) { return p != nullptr && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Validates sizes shared by sfa_fwd / sfa_bwd and builds the virtual-problem geometry.
+hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, int window,
+                      SfaGeom* g) {
+  if (B <= 0 || L <= 0 || n <= 0 || Hq <= 0 || Hkv <= 0 || Dh <= 0) return HD_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return HD_ERR_INVALID_ARG;
+  if (mode != SFA_WITHIN && mode != SFA_CROSS && mode != SFA_LOCAL) return HD_ERR_INVALID_ARG;
+  if (mode == SFA_LOCAL && window <= 0) return HD_ERR_INVALID_ARG;
+  if (Dh != 64 && Dh != 128) return HD_ERR_UNSUPPORTED;
+  const long long nL = (long long)n * L;
+  // Every row index, head product and tile count must fit the kernels' int math.
+  if (nL > (1LL << 30) || (long long)B * nL * Hq > (1LL << 31) / 2) return HD_ERR_UNSUPPORTED;
+  g->B = B;
+  g->nL = (int)nL;
+  g->Hq = Hq;
+  g->Hkv = Hkv;
+  g->n = n;
+  if (mode == SFA_WITHIN) {
+    g->Lv = L;
+    g->ns = n;
+    g->rs = n;
+    g->window = 0;
+  } else {
+    g->Lv = (int)nL;
+    g->ns = 1;
+    g->rs = 1;
+    g->window = mode == SFA_LOCAL ? window : 0;
+  }
+  return HD_OK;
+}
+
+float resolve_scale(float s, int Dh) { return s > 0.f ? s : 1.0f / sqrtf((float)Dh); }
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then fp32 delta [B][Hq][nL].
+struct BwdWs {
+  float* dq;
+  float* delta;
+};
+
+hd_status_t split_ws(const SfaGeom& g, int Dh, void* ws, size_t bytes, BwdWs* out) {
+  const size_t rows = (size_t)g.B * g.nL * g.Hq;
+  const size_t need = align256(rows * Dh * sizeof(float)) + align256(rows * sizeof(float));
+  if (ws == nullptr || bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return HD_ERR_WORKSPACE;
+  out->dq = static_cast<float*>(ws);
+  out->delta = reinterpret_cast<float*>(static_cast<char*>(ws) + align256(rows * Dh * sizeof(float)));
+  return HD_OK;
+}
+
+hd_status_t cuda_status(cudaError_t e) { return e == cudaSuccess ? HD_OK : HD_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L, int n,
+                            int V, int D, int32_t* dev_status, cudaStream_t stream) {
+  if (!aligned16(tables) || !aligned16(out) || ids == nullptr) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || n <= 0 || V <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  return hdsfa::launch_expand_embed(tables, ids, out, B, L, n, V, D, dev_status, stream) == cudaSuccess
+             ? HD_OK
+             : HD_ERR_CUDA;
+}
+
+hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
+                    int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode,
+                    int window, int32_t* dev_status, cudaStream_t stream) {
+  (void)dev_status;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
+    return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
+  if (st != HD_OK) return st;
+  const float scale = resolve_scale(softmax_scale, Dh);
+  return hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream) == cudaSuccess ? HD_OK
+                                                                                       : HD_ERR_CUDA;
+}
+
+size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode) {
+  SfaGeom g;
+  if (make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g) != HD_OK) return 0;
+  const size_t rows = (size_t)B * g.nL * Hq;
+  return align256(rows * Dh * sizeof(float)) + align256(rows * sizeof(float));
+}
+
+hd_status_t sfa_bwd_prep(const void* o, const void* dout, int B, int L, int n, int Hq, int Hkv,
+                         int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
+                         cudaStream_t stream) {
+  if (!aligned16(o) || !aligned16(dout)) return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
+  if (st != HD_OK) return st;
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  return cuda_status(hdsfa::launch_sfa_bwd_prep(o, dout, ws.delta, ws.dq, g, Dh, stream));
+}
+
+hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const float* lse,
+                         const void* dout, void* dk, void* dv, int B, int L, int n, int Hq, int Hkv,
+                         int Dh, float softmax_scale, sfa_mode_t mode, int window, void* workspace,
+                         size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream) {
+  (void)dev_status;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(lse) || !aligned16(dout) ||
+      !aligned16(dk) || !aligned16(dv))
+    return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
+  if (st != HD_OK) return st;
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  return cuda_status(hdsfa::launch_sfa_bwd_main_mma(q, k, v, lse, dout, dk, dv, ws.delta, ws.dq, g,
+                                                    Dh, resolve_scale(softmax_scale, Dh), stream));
+}
+
+hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
+                             float softmax_scale, sfa_mode_t mode, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+  if (!aligned16(dq)) return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
+  if (st != HD_OK) return st;
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  return cuda_status(hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, g, Dh,
+                                                    resolve_scale(softmax_scale, Dh), stream));
+}
+
+hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                    const void* dout, void* dq, void* dk, void* dv, int B, int L, int n, int Hq,
+                    int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
+                    void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                    cudaStream_t stream) {
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
+      !aligned16(dout) || !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+    return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
+  if (st != HD_OK) return st;
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  st = sfa_bwd_prep(o, dout, B, L, n, Hq, Hkv, Dh, mode, workspace, workspace_bytes, stream);
+  if (st != HD_OK) return st;
+  st = sfa_bwd_main(q, k, v, lse, dout, dk, dv, B, L, n, Hq, Hkv, Dh, softmax_scale, mode, window,
+                    workspace, workspace_bytes, dev_status, stream);
+  if (st != HD_OK) return st;
+  return sfa_bwd_finalize(dq, B, L, n, Hq, Hkv, Dh, softmax_scale, mode, workspace,
+                          workspace_bytes, stream);
+}
+
+const char* hd_status_string(hd_status_t s) {
+  switch (s) {
+    case HD_OK: return "HD_OK";
+    case HD_ERR_INVALID_ARG: return "HD_ERR_INVALID_ARG: invalid argument";
+    case HD_ERR_UNSUPPORTED: return "HD_ERR_UNSUPPORTED: configuration not supported";
+    case HD_ERR_CUDA: return "HD_ERR_CUDA: CUDA launch or runtime error";
+    case HD_ERR_WORKSPACE: return "HD_ERR_WORKSPACE: workspace missing, misaligned or too small";
+    case HD_ERR_TIMEOUT: return "HD_ERR_TIMEOUT: bounded device wait expired";
+    case HD_ERR_INDEX: return "HD_ERR_INDEX: index out of range";
+  }
+  return "unknown hd_status_t";
+}
+
+}  // extern "C"

@@ -1,0 +1,554 @@
+// Stream-Factorized Attention forward and backward on warp-level mma.sync
+// (m16n8k16 bf16, fp32 accumulate): FlashAttention-2-style tiles, cp.async
+// double buffering, XOR-swizzled shared memory.
+//
+// Each CTA works on one virtual causal problem (see SfaGeom): WITHIN mode gives
+// one problem per stream (rows p = r*n + s, Eq. 4), so a query tile visits only
+// its own stream's key tiles; CROSS gives one causal problem over nL positions
+// (Fig. 2a); LOCAL adds the window bound (Fig. 2b).  Key tiles beyond the causal
+// diagonal (or before the window) are never visited; only tiles that straddle a
+// mask edge are masked in registers.
+#include "common.cuh"
+
+namespace hdsfa {
+
+typedef __nv_bfloat16 bf16;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int BM = 64, BN = 64, NT = 128;
+
+struct MmaFwdArgs {
+  const bf16* q;
+  const bf16* k;
+  const bf16* v;
+  bf16* o;
+  float* lse;
+  SfaGeom g;
+  float scale_log2;
+};
+
+struct MmaBwdArgs {
+  const bf16* q;
+  const bf16* k;
+  const bf16* v;
+  const bf16* dout;
+  const float* lse;
+  const float* delta;  // [B][Hq][nL] rowsum(dO * O)
+  float* dq_acc;       // [B][nL][Hq][Dh] fp32, pre-zeroed; gets sum dS K (unscaled)
+  bf16* dk;
+  bf16* dv;
+  SfaGeom g;
+  float scale;
+  float scale_log2;
+};
+
+// rows [r0, r0 + ROWS) of a [*][DH] row set (row stride rstride elements) -> swizzled smem.
+template <int DH, int ROWS>
+HD_DEVINLINE void load_rows(bf16* s, const bf16* base, long long rstride, int r0, int Lv, int tid) {
+  constexpr int CPR = DH / 8;
+#pragma unroll
+  for (int i = tid; i < ROWS * CPR; i += NT) {
+    const int r = i / CPR, c = i % CPR;
+    const int gr = r0 + r;
+    const bool ok = gr < Lv;
+    const bf16* src = base + (long long)(ok ? gr : 0) * rstride + c * 8;
+    cp_async_16(smem_u32(s + swz<DH>(r, c * 8)), src, ok);
+  }
+}
+
+HD_DEVINLINE bool visible(int r, int c, int Lv, int window) {
+  return c <= r && c < Lv && (window <= 0 || r - c < window);
+}
+
+// ----------------------------------------------------------------- forward
+template <int DH>
+__global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  bf16* sQ = reinterpret_cast<bf16*>(smem_raw);  // [BM][DH]
+  bf16* sK = sQ + BM * DH;                        // [2][BN][DH]
+  bf16* sV = sK + 2 * BN * DH;                    // [2][BN][DH]
+  const SfaGeom G = a.g;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int ntile = (G.Lv + BM - 1) / BM;
+  const int mt = ntile - 1 - (int)blockIdx.x;  // longest rows first
+  const int m0 = mt * BM;
+  const int h = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
+  const int kvh = h / (G.Hq / G.Hkv);
+  const long long q_rs = (long long)G.rs * G.Hq * DH, kv_rs = (long long)G.rs * G.Hkv * DH;
+  const bf16* qb = a.q + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+  const bf16* kb = a.k + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  const bf16* vb = a.v + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  const int n_lo = G.window > 0 ? max(0, m0 - G.window + 1) / BN : 0;
+  const int n_hi = mt;  // BM == BN: the diagonal tile
+
+  load_rows<DH, BM>(sQ, qb, q_rs, m0, G.Lv, tid);
+  load_rows<DH, BN>(sK, kb, kv_rs, n_lo * BN, G.Lv, tid);
+  load_rows<DH, BN>(sV, vb, kv_rs, n_lo * BN, G.Lv, tid);
+  cp_async_commit();
+
+  uint32_t qf[DH / 16][4];
+  float oacc[DH / 8][4];
+#pragma unroll
+  for (int i = 0; i < DH / 8; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
+  float mx[2] = {-INFINITY, -INFINITY}, lsum[2] = {0.f, 0.f};
+  const int g4 = lane >> 2, t4 = lane & 3;
+  const int r_lo = m0 + warp * 16 + g4;
+
+  for (int nt_i = n_lo; nt_i <= n_hi; ++nt_i) {
+    const int buf = (nt_i - n_lo) & 1;
+    cp_async_wait<0>();
+    __syncthreads();
+    if (nt_i == n_lo) {
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk)
+        ldsm_x4(smem_u32(sQ + swz<DH>(warp * 16 + (lane & 15), kk * 16 + (lane >> 4) * 8)),
+                qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+    }
+    if (nt_i < n_hi) {
+      load_rows<DH, BN>(sK + (buf ^ 1) * BN * DH, kb, kv_rs, (nt_i + 1) * BN, G.Lv, tid);
+      load_rows<DH, BN>(sV + (buf ^ 1) * BN * DH, vb, kv_rs, (nt_i + 1) * BN, G.Lv, tid);
+      cp_async_commit();
+    }
+    const bf16* cK = sK + buf * BN * DH;
+    const bf16* cV = sV + buf * BN * DH;
+    const int n0 = nt_i * BN;
+
+    float sacc[BN / 8][4];
+#pragma unroll
+    for (int i = 0; i < BN / 8; ++i) sacc[i][0] = sacc[i][1] = sacc[i][2] = sacc[i][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < DH / 16; ++kk) {
+#pragma unroll
+      for (int np = 0; np < BN / 16; ++np) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(smem_u32(cK + swz<DH>(np * 16 + (lane & 7) + (lane >> 4) * 8,
+                                      kk * 16 + ((lane >> 3) & 1) * 8)),
+                b0, b1, b2, b3);
+        mma_bf16_16816(sacc[2 * np], qf[kk], b0, b1);
+        mma_bf16_16816(sacc[2 * np + 1], qf[kk], b2, b3);
+      }
+    }
+    const bool need_mask = (nt_i == n_hi) || G.window > 0;
+    float tmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int i = 0; i < BN / 8; ++i) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float x = sacc[i][e] * a.scale_log2;
+        if (need_mask) {
+          const int r = r_lo + (e >> 1) * 8, c = n0 + i * 8 + 2 * t4 + (e & 1);
+          if (!visible(r, c, G.Lv, G.window)) x = -INFINITY;
+        }
+        sacc[i][e] = x;
+        tmax[e >> 1] = fmaxf(tmax[e >> 1], x);
+      }
+    }
+    float corr[2];
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      tmax[hh] = fmaxf(tmax[hh], __shfl_xor_sync(0xffffffffu, tmax[hh], 1));
+      tmax[hh] = fmaxf(tmax[hh], __shfl_xor_sync(0xffffffffu, tmax[hh], 2));
+      const float mnew = fmaxf(mx[hh], tmax[hh]);
+      const float muse = (mnew == -INFINITY) ? 0.f : mnew;
+      corr[hh] = exp2f(mx[hh] - muse);
+      mx[hh] = mnew;
+      lsum[hh] *= corr[hh];
+      tmax[hh] = muse;
+    }
+#pragma unroll
+    for (int i = 0; i < BN / 8; ++i) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float p = exp2f(sacc[i][e] - tmax[e >> 1]);
+        sacc[i][e] = p;
+        lsum[e >> 1] += p;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < DH / 8; ++i) {
+      oacc[i][0] *= corr[0];
+      oacc[i][1] *= corr[0];
+      oacc[i][2] *= corr[1];
+      oacc[i][3] *= corr[1];
+    }
+#pragma unroll
+    for (int kk = 0; kk < BN / 16; ++kk) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16(sacc[2 * kk][0], sacc[2 * kk][1]);
+      pa[1] = pack_bf16(sacc[2 * kk][2], sacc[2 * kk][3]);
+      pa[2] = pack_bf16(sacc[2 * kk + 1][0], sacc[2 * kk + 1][1]);
+      pa[3] = pack_bf16(sacc[2 * kk + 1][2], sacc[2 * kk + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < DH / 16; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(smem_u32(cV + swz<DH>(kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8,
+                                        dp * 16 + (lane >> 4) * 8)),
+                  b0, b1, b2, b3);
+        mma_bf16_16816(oacc[2 * dp], pa, b0, b1);
+        mma_bf16_16816(oacc[2 * dp + 1], pa, b2, b3);
+      }
+    }
+  }
+
+  // epilogue: normalise, stage through shared memory, coalesced 16-byte stores
+#pragma unroll
+  for (int hh = 0; hh < 2; ++hh) {
+    lsum[hh] += __shfl_xor_sync(0xffffffffu, lsum[hh], 1);
+    lsum[hh] += __shfl_xor_sync(0xffffffffu, lsum[hh], 2);
+  }
+  const float inv0 = 1.f / lsum[0], inv1 = 1.f / lsum[1];
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < DH / 8; ++i) {
+    const int row = warp * 16 + g4, col = i * 8 + 2 * t4;
+    *reinterpret_cast<uint32_t*>(sQ + swz<DH>(row, col)) = pack_bf16(oacc[i][0] * inv0, oacc[i][1] * inv0);
+    *reinterpret_cast<uint32_t*>(sQ + swz<DH>(row + 8, col)) = pack_bf16(oacc[i][2] * inv1, oacc[i][3] * inv1);
+  }
+  if (t4 == 0) {
+    float* lrow = a.lse + ((long long)b * G.Hq + h) * G.nL + s;
+    if (r_lo < G.Lv) lrow[(long long)r_lo * G.rs] = (mx[0] + log2f(lsum[0])) * kLn2;
+    if (r_lo + 8 < G.Lv) lrow[(long long)(r_lo + 8) * G.rs] = (mx[1] + log2f(lsum[1])) * kLn2;
+  }
+  __syncthreads();
+  bf16* ob = a.o + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+  constexpr int CPR = DH / 8;
+  for (int i = tid; i < BM * CPR; i += NT) {
+    const int r = i / CPR, c = i % CPR;
+    if (m0 + r < G.Lv)
+      *reinterpret_cast<uint4*>(ob + (long long)(m0 + r) * q_rs + c * 8) =
+          *reinterpret_cast<const uint4*>(sQ + swz<DH>(r, c * 8));
+  }
+}
+
+// ----------------------------------------------------------------- backward
+// delta[b][h][p] = sum_d dO * O (fp32), and zero the fp32 dQ accumulator row.
+template <int DH>
+__global__ void __launch_bounds__(256) sfa_bwd_pre_kernel(const bf16* __restrict__ o,
+                                                          const bf16* __restrict__ dout,
+                                                          float* __restrict__ delta,
+                                                          float* __restrict__ dq_acc, int B,
+                                                          int nL, int Hq) {
+  const int lane = threadIdx.x & 31;
+  const long long row = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // (b, p, h)
+  if (row >= (long long)B * nL * Hq) return;
+  float acc = 0.f;
+  if (lane < DH / 8) {
+    const uint4 x = *reinterpret_cast<const uint4*>(o + row * DH + lane * 8);
+    const uint4 y = *reinterpret_cast<const uint4*>(dout + row * DH + lane * 8);
+    const bf16* xa = reinterpret_cast<const bf16*>(&x);
+    const bf16* ya = reinterpret_cast<const bf16*>(&y);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc += __bfloat162float(xa[i]) * __bfloat162float(ya[i]);
+  }
+#pragma unroll
+  for (int off = 16; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  float4* dqr = reinterpret_cast<float4*>(dq_acc + row * DH);
+  for (int c = lane; c < DH / 4; c += 32) dqr[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (lane == 0) {
+    const long long h = row % Hq, bp = row / Hq, p = bp % nL, b = bp / nL;
+    delta[(b * Hq + h) * nL + p] = acc;
+  }
+}
+
+// dq = scale * dq_acc, fp32 -> bf16 (round to nearest even), 8 elements per thread.
+__global__ void __launch_bounds__(256) sfa_bwd_post_kernel(const float* __restrict__ dq_acc,
+                                                           bf16* __restrict__ dq, long long n8,
+                                                           float scale) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n8) return;
+  const float4 a = reinterpret_cast<const float4*>(dq_acc)[2 * i];
+  const float4 c = reinterpret_cast<const float4*>(dq_acc)[2 * i + 1];
+  uint4 r;
+  r.x = pack_bf16(a.x * scale, a.y * scale);
+  r.y = pack_bf16(a.z * scale, a.w * scale);
+  r.z = pack_bf16(c.x * scale, c.y * scale);
+  r.w = pack_bf16(c.z * scale, c.w * scale);
+  reinterpret_cast<uint4*>(dq)[i] = r;
+}
+
+// One CTA per (key tile j, b, K/V head g, stream s).  It keeps dK_j, dV_j in
+// registers while looping over the group's query heads and the query tiles that
+// can see tile j; dQ contributions go to the fp32 accumulator with atomics.
+// Warp w owns key rows [16w, 16w + 16) of the tile for S^T, dP^T, dK, dV.
+template <int DH>
+__global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  bf16* sK = reinterpret_cast<bf16*>(smem_raw);  // [BN][DH]
+  bf16* sV = sK + BN * DH;                        // [BN][DH]
+  bf16* sQ = sV + BN * DH;                        // [2][BM][DH]
+  bf16* sdO = sQ + 2 * BM * DH;                   // [2][BM][DH]
+  bf16* sdS = sdO + 2 * BM * DH;                  // [BN][BM]  (dS^T, key-major)
+  float* sL = reinterpret_cast<float*>(sdS + BN * BM);  // [2][BM] lse * log2(e)
+  float* sD = sL + 2 * BM;                               // [2][BM] delta
+
+  const SfaGeom G = a.g;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g4 = lane >> 2, t4 = lane & 3;
+  const int ntile = (G.Lv + BM - 1) / BM;
+  const int j = blockIdx.x;  // key tile; tile 0 sees the most query tiles, so it starts first
+  const int n0 = j * BN;
+  const int kvh = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
+  const int grp = G.Hq / G.Hkv;
+  int mi_hi = ntile - 1;
+  if (G.window > 0) mi_hi = min(mi_hi, (n0 + BN - 1 + G.window - 1) / BM);
+  const int nq = mi_hi - j + 1;
+  const int total = grp * nq;
+  const long long q_rs = (long long)G.rs * G.Hq * DH, kv_rs = (long long)G.rs * G.Hkv * DH;
+  const bf16* kb = a.k + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  const bf16* vb = a.v + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+
+  auto q_base = [&](const bf16* t, int h) {
+    return t + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+  };
+  auto row_terms = [&](int it, int r, float& l2, float& dl) {
+    const int h = kvh * grp + it / nq, m0 = (j + it % nq) * BM;
+    const long long idx = ((long long)b * G.Hq + h) * G.nL + (long long)(m0 + r) * G.rs + s;
+    const bool ok = m0 + r < G.Lv;
+    l2 = ok ? a.lse[idx] * kLog2e : 0.f;
+    dl = ok ? a.delta[idx] : 0.f;
+  };
+
+  load_rows<DH, BN>(sK, kb, kv_rs, n0, G.Lv, tid);
+  load_rows<DH, BN>(sV, vb, kv_rs, n0, G.Lv, tid);
+  {
+    const int h = kvh * grp;
+    load_rows<DH, BM>(sQ, q_base(a.q, h), q_rs, j * BM, G.Lv, tid);
+    load_rows<DH, BM>(sdO, q_base(a.dout, h), q_rs, j * BM, G.Lv, tid);
+  }
+  cp_async_commit();
+  if (tid < BM) {
+    float l2, dl;
+    row_terms(0, tid, l2, dl);
+    sL[tid] = l2;
+    sD[tid] = dl;
+  }
+
+  float dK[DH / 8][4], dV[DH / 8][4];
+#pragma unroll
+  for (int i = 0; i < DH / 8; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) dK[i][e] = dV[i][e] = 0.f;
+
+  for (int it = 0; it < total; ++it) {
+    const int buf = it & 1;
+    cp_async_wait<0>();
+    __syncthreads();
+    const bool has_next = it + 1 < total;
+    float nl2 = 0.f, ndl = 0.f;
+    if (has_next) {
+      const int h1 = kvh * grp + (it + 1) / nq, m1 = (j + (it + 1) % nq) * BM;
+      load_rows<DH, BM>(sQ + (buf ^ 1) * BM * DH, q_base(a.q, h1), q_rs, m1, G.Lv, tid);
+      load_rows<DH, BM>(sdO + (buf ^ 1) * BM * DH, q_base(a.dout, h1), q_rs, m1, G.Lv, tid);
+      cp_async_commit();
+      if (tid < BM) row_terms(it + 1, tid, nl2, ndl);
+    }
+    const int h = kvh * grp + it / nq;
+    const int m0 = (j + it % nq) * BM;
+    const bf16* cQ = sQ + buf * BM * DH;
+    const bf16* cdO = sdO + buf * BM * DH;
+    const float* cL = sL + buf * BM;
+    const float* cD = sD + buf * BM;
+
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      float sacc[4][4], dpacc[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sacc[i][e] = dpacc[i][e] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk) {
+        uint32_t ka[4], va[4];
+        ldsm_x4(smem_u32(sK + swz<DH>(warp * 16 + (lane & 15), kk * 16 + (lane >> 4) * 8)),
+                ka[0], ka[1], ka[2], ka[3]);
+        ldsm_x4(smem_u32(sV + swz<DH>(warp * 16 + (lane & 15), kk * 16 + (lane >> 4) * 8)),
+                va[0], va[1], va[2], va[3]);
+#pragma unroll
+        for (int np = 0; np < 2; ++np) {
+          const int qr = half * 32 + np * 16 + (lane & 7) + (lane >> 4) * 8;
+          const int qc = kk * 16 + ((lane >> 3) & 1) * 8;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(smem_u32(cQ + swz<DH>(qr, qc)), b0, b1, b2, b3);
+          mma_bf16_16816(sacc[2 * np], ka, b0, b1);
+          mma_bf16_16816(sacc[2 * np + 1], ka, b2, b3);
+          ldsm_x4(smem_u32(cdO + swz<DH>(qr, qc)), b0, b1, b2, b3);
+          mma_bf16_16816(dpacc[2 * np], va, b0, b1);
+          mma_bf16_16816(dpacc[2 * np + 1], va, b2, b3);
+        }
+      }
+      // P^T and dS^T for rows (key) kr, columns (query) qc
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int kr = n0 + warp * 16 + g4 + (e >> 1) * 8;
+          const int ql = half * 32 + i * 8 + 2 * t4 + (e & 1);
+          const int qr = m0 + ql;
+          float p = 0.f;
+          if (visible(qr, kr, G.Lv, G.window) && qr < G.Lv)
+            p = exp2f(sacc[i][e] * a.scale_log2 - cL[ql]);
+          sacc[i][e] = p;
+          dpacc[i][e] = p * (dpacc[i][e] - cD[ql]);
+        }
+      }
+#pragma unroll
+      for (int kk = 0; kk < 2; ++kk) {
+        uint32_t pa[4], da[4];
+        pa[0] = pack_bf16(sacc[2 * kk][0], sacc[2 * kk][1]);
+        pa[1] = pack_bf16(sacc[2 * kk][2], sacc[2 * kk][3]);
+        pa[2] = pack_bf16(sacc[2 * kk + 1][0], sacc[2 * kk + 1][1]);
+        pa[3] = pack_bf16(sacc[2 * kk + 1][2], sacc[2 * kk + 1][3]);
+        da[0] = pack_bf16(dpacc[2 * kk][0], dpacc[2 * kk][1]);
+        da[1] = pack_bf16(dpacc[2 * kk][2], dpacc[2 * kk][3]);
+        da[2] = pack_bf16(dpacc[2 * kk + 1][0], dpacc[2 * kk + 1][1]);
+        da[3] = pack_bf16(dpacc[2 * kk + 1][2], dpacc[2 * kk + 1][3]);
+        const int qrow = half * 32 + kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+        for (int dp = 0; dp < DH / 16; ++dp) {
+          const int dcol = dp * 16 + (lane >> 4) * 8;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(smem_u32(cdO + swz<DH>(qrow, dcol)), b0, b1, b2, b3);
+          mma_bf16_16816(dV[2 * dp], pa, b0, b1);
+          mma_bf16_16816(dV[2 * dp + 1], pa, b2, b3);
+          ldsm_x4_t(smem_u32(cQ + swz<DH>(qrow, dcol)), b0, b1, b2, b3);
+          mma_bf16_16816(dK[2 * dp], da, b0, b1);
+          mma_bf16_16816(dK[2 * dp + 1], da, b2, b3);
+        }
+        // dS^T (bf16) to shared memory for the dQ product
+        const int krow = warp * 16 + g4;
+        const int qcol = half * 32 + kk * 16 + 2 * t4;
+        *reinterpret_cast<uint32_t*>(sdS + swz<BM>(krow, qcol)) = da[0];
+        *reinterpret_cast<uint32_t*>(sdS + swz<BM>(krow + 8, qcol)) = da[1];
+        *reinterpret_cast<uint32_t*>(sdS + swz<BM>(krow, qcol + 8)) = da[2];
+        *reinterpret_cast<uint32_t*>(sdS + swz<BM>(krow + 8, qcol + 8)) = da[3];
+      }
+    }
+    __syncthreads();
+    // dQ[q rows of warp] += dS K  (unscaled; the post kernel applies the scale)
+    {
+      float* dqb = a.dq_acc + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+      const int qa = m0 + warp * 16 + g4;
+#pragma unroll
+      for (int dh = 0; dh < 2; ++dh) {
+        float qacc[DH / 16][4];
+#pragma unroll
+        for (int i = 0; i < DH / 16; ++i) qacc[i][0] = qacc[i][1] = qacc[i][2] = qacc[i][3] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          uint32_t aa[4];
+          ldsm_x4_t(smem_u32(sdS + swz<BM>(kk * 16 + (lane & 7) + (lane >> 4) * 8,
+                                           warp * 16 + ((lane >> 3) & 1) * 8)),
+                    aa[0], aa[1], aa[2], aa[3]);
+#pragma unroll
+          for (int dp = 0; dp < DH / 32; ++dp) {
+            uint32_t b0, b1, b2, b3;
+            ldsm_x4_t(smem_u32(sK + swz<DH>(kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8,
+                                            dh * (DH / 2) + dp * 16 + (lane >> 4) * 8)),
+                      b0, b1, b2, b3);
+            mma_bf16_16816(qacc[2 * dp], aa, b0, b1);
+            mma_bf16_16816(qacc[2 * dp + 1], aa, b2, b3);
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < DH / 16; ++i) {
+          const int col = dh * (DH / 2) + i * 8 + 2 * t4;
+          if (qa < G.Lv)
+            atomicAdd(reinterpret_cast<float2*>(dqb + (long long)qa * q_rs + col),
+                      make_float2(qacc[i][0], qacc[i][1]));
+          if (qa + 8 < G.Lv)
+            atomicAdd(reinterpret_cast<float2*>(dqb + (long long)(qa + 8) * q_rs + col),
+                      make_float2(qacc[i][2], qacc[i][3]));
+        }
+      }
+    }
+    if (has_next && tid < BM) {
+      sL[(buf ^ 1) * BM + tid] = nl2;
+      sD[(buf ^ 1) * BM + tid] = ndl;
+    }
+  }
+
+  // epilogue: dK *= scale, write dK and dV rows of this key tile
+  bf16* dkb = a.dk + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  bf16* dvb = a.dv + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  const int kr = n0 + warp * 16 + g4;
+#pragma unroll
+  for (int i = 0; i < DH / 8; ++i) {
+    const int col = i * 8 + 2 * t4;
+    if (kr < G.Lv) {
+      *reinterpret_cast<uint32_t*>(dkb + (long long)kr * kv_rs + col) =
+          pack_bf16(dK[i][0] * a.scale, dK[i][1] * a.scale);
+      *reinterpret_cast<uint32_t*>(dvb + (long long)kr * kv_rs + col) = pack_bf16(dV[i][0], dV[i][1]);
+    }
+    if (kr + 8 < G.Lv) {
+      *reinterpret_cast<uint32_t*>(dkb + (long long)(kr + 8) * kv_rs + col) =
+          pack_bf16(dK[i][2] * a.scale, dK[i][3] * a.scale);
+      *reinterpret_cast<uint32_t*>(dvb + (long long)(kr + 8) * kv_rs + col) =
+          pack_bf16(dV[i][2], dV[i][3]);
+    }
+  }
+}
+
+// ----------------------------------------------------------------- launchers
+template <int DH>
+static cudaError_t fwd_impl(const MmaFwdArgs& a, cudaStream_t st) {
+  const int smem = (BM + 4 * BN) * DH * (int)sizeof(bf16);
+  cudaError_t e = cudaFuncSetAttribute(sfa_fwd_mma_kernel<DH>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((a.g.Lv + BM - 1) / BM, a.g.Hq * a.g.ns, a.g.B);
+  sfa_fwd_mma_kernel<DH><<<grid, NT, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
+                               const SfaGeom& g, int Dh, float scale, cudaStream_t st) {
+  MmaFwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (bf16*)o, lse, g, scale * kLog2e};
+  return Dh == 64 ? fwd_impl<64>(a, st) : fwd_impl<128>(a, st);
+}
+
+cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, float* delta_ws, float* dq_ws,
+                                const SfaGeom& g, int Dh, cudaStream_t st) {
+  const long long rows = (long long)g.B * g.nL * g.Hq;
+  const unsigned blocks = (unsigned)((rows * 32 + 255) / 256);
+  if (Dh == 64)
+    sfa_bwd_pre_kernel<64><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, delta_ws,
+                                                  dq_ws, g.B, g.nL, g.Hq);
+  else
+    sfa_bwd_pre_kernel<128><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, delta_ws,
+                                                   dq_ws, g.B, g.nL, g.Hq);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const float* lse,
+                                    const void* dout, void* dk, void* dv, const float* delta_ws,
+                                    float* dq_ws, const SfaGeom& g, int Dh, float scale,
+                                    cudaStream_t st) {
+  MmaBwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)dout, lse, delta_ws,
+               dq_ws, (bf16*)dk, (bf16*)dv, g, scale, scale * kLog2e};
+  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.ns, g.B);
+  auto smem_of = [](int dh) {
+    return (2 * BN * dh + 4 * BM * dh + BN * BM) * (int)sizeof(bf16) + 4 * BM * (int)sizeof(float);
+  };
+  cudaError_t e;
+  if (Dh == 64) {
+    const int smem = smem_of(64);
+    e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    sfa_bwd_mma_kernel<64><<<grid, NT, smem, st>>>(a);
+  } else {
+    const int smem = smem_of(128);
+    e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    sfa_bwd_mma_kernel<128><<<grid, NT, smem, st>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
+                                    float scale, cudaStream_t st) {
+  const long long n8 = (long long)g.B * g.nL * g.Hq * Dh / 8;
+  sfa_bwd_post_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dq_ws, (bf16*)dq, n8, scale);
+  return cudaGetLastError();
+}
+
+}  // namespace hdsfa

@@ -41,10 +41,15 @@ SHAPES = {
 def _randn(shape, seed: int, std: float = 1.0) -> torch.Tensor:
     g = torch.Generator(device="cpu")
     g.manual_seed(seed)
-    x = torch.randn(shape, generator=g, dtype=torch.float32)
-    if std != 1.0:
-        x.mul_(std)
-    return x.to(torch.bfloat16)
+    out = torch.empty(shape, dtype=torch.bfloat16)
+    flat = out.view(-1)
+    chunk = 1 << 26
+    for i in range(0, flat.numel(), chunk):
+        x = torch.randn(min(chunk, flat.numel() - i), generator=g, dtype=torch.float32)
+        if std != 1.0:
+            x.mul_(std)
+        flat[i:i + x.numel()] = x.to(torch.bfloat16)
+    return out
 
 
 def attn_inputs(s: AttnShape, seed: int = 0, with_grad: bool = True):

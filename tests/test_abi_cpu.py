@@ -1,0 +1,93 @@
+"""Host-only checks of the C ABI: the library builds, loads and exports every
+symbol include/hdsfa.h declares; argument validation answers before anything is
+launched (no GPU needed, no compute call reaches a kernel)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_08186_gb300 import binding, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "hdsfa.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return binding.lib()
+
+
+def _declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*([a-z_][a-z0-9_]*)\s*\(",
+                                 src, flags=re.M)))
+
+
+def test_header_declares_the_entry_points():
+    names = _declared_functions()
+    for want in ("hd_expand_embed", "sfa_fwd", "sfa_bwd", "sfa_bwd_workspace_bytes", "hd_status_string"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    for code in range(7):
+        assert binding.hd_status_string(code).startswith("HD_")
+    assert "unknown" in binding.hd_status_string(99)
+
+
+FAKE = 1 << 20  # 16-byte aligned non-null address; never dereferenced (validation fails first)
+
+
+def _fwd(lib, B=1, L=8, n=2, Hq=4, Hkv=2, Dh=64, mode=0, window=0, ptr=FAKE):
+    P = ctypes.c_void_p
+    return lib.sfa_fwd(P(ptr), P(ptr), P(ptr), P(ptr), P(ptr), B, L, n, Hq, Hkv, Dh, 0.0, mode,
+                       window, None, None)
+
+
+def test_fwd_validation(lib):
+    assert _fwd(lib, B=0) == 1
+    assert _fwd(lib, L=-1) == 1
+    assert _fwd(lib, n=0) == 1
+    assert _fwd(lib, Hq=6, Hkv=4) == 1          # Hq % Hkv != 0
+    assert _fwd(lib, mode=7) == 1
+    assert _fwd(lib, mode=2, window=0) == 1     # LOCAL needs a window
+    assert _fwd(lib, ptr=FAKE + 8) == 1         # misaligned
+    assert _fwd(lib, ptr=0) == 1                # null
+    assert _fwd(lib, Dh=96) == 2                # unsupported head dim
+    assert _fwd(lib, Dh=256) == 2
+
+
+def test_bwd_workspace_size(lib):
+    B, L, n, Hq, Hkv, Dh = 1, 100, 4, 8, 2, 128
+    ws = binding.sfa_bwd_workspace_bytes(B, L, n, Hq, Hkv, Dh, 0)
+    rows = B * n * L * Hq
+    assert ws >= rows * Dh * 4 + rows * 4
+    assert binding.sfa_bwd_workspace_bytes(0, L, n, Hq, Hkv, Dh, 0) == 0
+    assert binding.sfa_bwd_workspace_bytes(B, L, n, Hq, Hkv, 80, 0) == 0
+
+
+def test_bwd_validation(lib):
+    P = ctypes.c_void_p
+    a = [P(FAKE)] * 9
+    need = binding.sfa_bwd_workspace_bytes(1, 8, 2, 4, 2, 64, 0)
+    assert lib.sfa_bwd(*a, 1, 8, 2, 4, 2, 64, 0.0, 0, 0, None, 0, None, None) == 4           # no workspace
+    assert lib.sfa_bwd(*a, 1, 8, 2, 4, 2, 64, 0.0, 0, 0, P(FAKE), need - 1, None, None) == 4  # too small
+    assert lib.sfa_bwd(*a, 1, 8, 2, 4, 2, 64, 0.0, 0, 0, P(FAKE + 16), need, None, None) == 4  # not 256-aligned
+    assert lib.sfa_bwd(*a, 1, 8, 2, 5, 2, 64, 0.0, 0, 0, P(FAKE), need, None, None) == 1
+    assert lib.sfa_bwd(*a, 1, 8, 2, 4, 2, 32, 0.0, 0, 0, P(FAKE), need, None, None) == 2
+
+
+def test_expand_validation(lib):
+    P = ctypes.c_void_p
+    assert lib.hd_expand_embed(P(FAKE), P(FAKE), P(FAKE), 1, 4, 2, 16, 12, None, None) == 1  # D % 8
+    assert lib.hd_expand_embed(P(FAKE), P(FAKE), P(FAKE + 2), 1, 4, 2, 16, 16, None, None) == 1
+    assert lib.hd_expand_embed(P(FAKE), None, P(FAKE), 1, 4, 2, 16, 16, None, None) == 1
+    assert lib.hd_expand_embed(P(FAKE), P(FAKE), P(FAKE), 1, 4, 0, 16, 16, None, None) == 1

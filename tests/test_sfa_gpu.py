@@ -1,0 +1,139 @@
+"""GPU parity: the CUDA SFA forward/backward (through the C ABI) against the fp64 oracle.
+
+Small shapes compare every element; they span several 64/128-row tiles and end
+in ragged tails.  Full-size shapes (the Qwen3-8B-class and large-MoE-class
+layers, in the launch configuration the benchmark times) compare sampled rows
+the oracle computes one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_08186_gb300 import binding, build, inputs
+from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, WITHIN
+
+from parity import (assert_fwd_close, assert_grads_close, gpu_fwd, gpu_fwd_bwd, group_slices,
+                    max_abs, sample_rows, TOL_LSE, TOL_O)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    build.build()
+    binding.lib()
+
+
+def _full_case(s: AttnShape, mode, seed, window=0, scale=0.0):
+    q, k, v, do = inputs.attn_inputs(s, seed=seed)
+    o, lse, dq, dk, dv = gpu_fwd_bwd(q, k, v, do, s.n, mode, scale, window)
+    o_ref, lse_ref = oracle.sfa_fwd(q, k, v, s.n, mode, scale or None, window)
+    assert_fwd_close(o, lse, o_ref, lse_ref)
+    dq_r, dk_r, dv_r = oracle.sfa_bwd(q, k, v, do, s.n, mode, scale or None, window)
+    assert_grads_close([("dq", dq, dq_r), ("dk", dk, dk_r), ("dv", dv, dv_r)])
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_tiny_config(mode):
+    # B=1, L=64, n=2 (128 positions), Hq=Hkv=4, Dh=64, N(0,1) from seed 0.
+    _full_case(inputs.SHAPES["tiny"], mode, seed=0)
+
+
+SWEEP = [
+    # (B, L, n, Hq, Hkv, Dh)
+    (1, 100, 1, 4, 2, 128),
+    (2, 37, 2, 4, 4, 64),
+    (1, 130, 4, 4, 1, 128),
+    (1, 70, 8, 2, 2, 64),
+    (1, 200, 4, 4, 2, 128),
+]
+
+
+@pytest.mark.parametrize("shape", SWEEP)
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_sweep(shape, mode):
+    _full_case(AttnShape(*shape), mode, seed=11 + sum(shape))
+
+
+@pytest.mark.parametrize("window", [1, 50, 200])
+def test_local_window(window):
+    _full_case(AttnShape(1, 96, 4, 4, 2, 128), LOCAL, seed=5, window=window)
+
+
+@pytest.mark.parametrize("L,n", [(1, 1), (1, 4), (2, 3), (63, 1), (65, 1), (64, 2)])
+def test_edge_sizes(L, n):
+    for mode in (WITHIN, CROSS):
+        _full_case(AttnShape(1, L, n, 2, 1, 64), mode, seed=3)
+
+
+def test_explicit_scale_and_first_rows():
+    s = AttnShape(1, 40, 4, 2, 2, 128)
+    _full_case(s, WITHIN, seed=8, scale=0.05)
+    q, k, v = inputs.attn_inputs(s, seed=9, with_grad=False)
+    _, _, _, o, lse = gpu_fwd(q, k, v, s.n, WITHIN)
+    # the first position of each stream sees only itself: O = V exactly (bf16 round trip)
+    for p in range(s.n):
+        assert torch.equal(o[0, p].cpu(), v[0, p])
+
+
+def test_deterministic_forward():
+    s = AttnShape(1, 300, 4, 4, 2, 128)
+    q, k, v = inputs.attn_inputs(s, seed=12, with_grad=False)
+    a = gpu_fwd(q, k, v, s.n, CROSS)
+    b = gpu_fwd(q, k, v, s.n, CROSS)
+    assert torch.equal(a[3], b[3]) and torch.equal(a[4], b[4])
+
+
+# ------------------------------------------------------------ full-size layers
+def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
+    q, k, v, do = inputs.attn_inputs(s, seed=seed)
+    o, lse, dq, dk, dv = gpu_fwd_bwd(q, k, v, do, s.n, mode)
+    grp = s.Hq // s.Hkv
+    edges = [0, 1, 63, 64, 127, 128, s.nL // 2, s.nL - 129, s.nL - 2, s.nL - 1]
+    rows = sample_rows(s.B, s.Hq, s.nL, n_rows, seed, edges)
+    # forward rows and dQ rows, oracle per K/V group
+    for g in range(s.Hkv):
+        sel = rows[(rows[:, 1] // grp) == g]
+        if not len(sel):
+            continue
+        qg, kg, vg, dog = group_slices(q, k, v, do, g, grp)
+        loc = sel.copy()
+        loc[:, 1] -= g * grp
+        o_r, l_r = oracle.sfa_fwd_rows(qg, kg, vg, s.n, mode, loc)
+        dq_r, _, _ = oracle.sfa_bwd_q_rows(qg, kg, vg, dog, s.n, mode, loc)
+        o_g = o[sel[:, 0], sel[:, 2], sel[:, 1]]
+        l_g = lse[sel[:, 0], sel[:, 1], sel[:, 2]]
+        assert max_abs(o_g, o_r) <= TOL_O
+        assert max_abs(l_g, l_r) <= TOL_LSE
+        assert_grads_close([("dq rows", dq[sel[:, 0], sel[:, 2], sel[:, 1]], dq_r)])
+    # dK / dV rows of one group: keys in the last 384 positions (complete sums
+    # over every query row and head of the group that sees them)
+    g = s.Hkv - 1
+    gen = torch.Generator().manual_seed(seed + 1)
+    ps = sorted({int(x) for x in torch.randint(s.nL - 384, s.nL, (n_kv,), generator=gen)} | {s.nL - 1})
+    kvrows = np.array([[0, 0, p] for p in ps], dtype=np.int64)
+    qg, kg, vg, dog = group_slices(q, k, v, do, g, grp)
+    dk_r, dv_r = oracle.sfa_bwd_kv_rows(qg, kg, vg, dog, s.n, mode, kvrows)
+    assert_grads_close([("dk rows", dk[0, ps, g], dk_r), ("dv rows", dv[0, ps, g], dv_r)])
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_qwen3_8b_class_layer(mode):
+    # B=1, L=4096, n=4 (16384 positions), Hq=32, Hkv=8, Dh=128
+    _sampled_parity(inputs.SHAPES["qwen3_8b_n4"], mode, seed=1)
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_large_moe_class_layer(mode):
+    # B=1, L=8192, n=4 (32768 positions), Hq=64, Hkv=8, Dh=128
+    _sampled_parity(inputs.SHAPES["moe_large_n4"], mode, seed=21, n_rows=96, n_kv=24)
+
+
+@pytest.mark.parametrize("n", [1, 2, 8])
+def test_expansion_sweep_layers(n):
+    # the n sweep at L=4096, Hq=32, Hkv=8, Dh=128 (WITHIN; CROSS at n=8 is the largest)
+    s = AttnShape(1, 4096, n, 32, 8, 128)
+    _sampled_parity(s, WITHIN, seed=31 + n, n_rows=64, n_kv=16)
+    if n == 8:
+        _sampled_parity(s, CROSS, seed=41, n_rows=32, n_kv=8)
