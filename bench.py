@@ -355,6 +355,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-extras", action="store_true", help="skip CROSS layer, n sweep and CPU baseline")
+    ap.add_argument("--layer-only", choices=["within", "cross"], default=None,
+                    help="time only one attention layer (fwd + bwd, no gather / e2e / extras); "
+                         "the small case used for kernel profiles")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     ws, rank, local = dist_setup()
@@ -371,6 +374,15 @@ def main():
     barrier(ws)
     s = SHAPES[WORKLOAD]
     pk = peaks()
+    if args.layer_only:
+        mode = WITHIN if args.layer_only == "within" else CROSS
+        r = measure_layer(s, mode, dev, iters=args.steps, warmup=args.warmup)
+        fl = attn_flops(s, mode, FWD_FLOP + BWD_FLOP)
+        if rank == 0:
+            print(json.dumps({"layer": f"{WORKLOAD}_{args.layer_only}", "ms": r["step_s"] * 1e3,
+                              "tflops": fl / r["step_s"] / 1e12, "fwd_ms": r["fwd_s"] * 1e3,
+                              "bwd_main_ms": r["bwd_main_s"] * 1e3}), flush=True)
+        return
     hp = HotPath(s, WITHIN, dev, with_gather=True, seed=1)
     flops_step = attn_flops(s, WITHIN, FWD_FLOP + BWD_FLOP)
 
