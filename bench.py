@@ -262,27 +262,33 @@ def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2):
 
 
 # ---------------------------------------------------------------- ncu traffic record
-def kernel_source_hash() -> str:
-    h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2607_08186_gb300", "csrc")
-    for fn in sorted(os.listdir(csrc)):
-        if fn.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, fn), "rb") as f:
-                h.update(f.read())
-    return h.hexdigest()[:16]
+# ABI phase -> (kernel symbol, source file) of the implementation the library runs.
+KERNEL_OF = {
+    "sfa_fwd": ("hdsfa::tcfwd::fwd_kernel<128>", "sfa_fwd_tc.cu"),
+    "sfa_bwd_main": ("hdsfa::sfa_bwd_mma_kernel<128>", "sfa_mma.cu"),
+}
+if os.environ.get("HDSFA_KERNELS") == "mma":
+    KERNEL_OF["sfa_fwd"] = ("hdsfa::sfa_fwd_mma_kernel<128>", "sfa_mma.cu")
 
 
-def traffic_record(kernel: str):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it was
-    taken on the current kernel sources (else None)."""
+def source_hash(fname: str) -> str:
+    with open(os.path.join(ROOT, "paper_2607_08186_gb300", "csrc", fname), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def traffic_record(phase: str):
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
+    kernel behind `phase`, from profiles/traffic.md, if it was captured on the
+    current source of that kernel's file (else None)."""
+    sym, fname = KERNEL_OF[phase]
     path = os.path.join(ROOT, "profiles", "traffic.md")
     if not os.path.exists(path):
         return None
-    txt = open(path).read()
-    m = re.search(rf"^\| {re.escape(kernel)} \| ([0-9a-f]+) \| ([0-9.e+]+) \|", txt, flags=re.M)
-    if not m or m.group(1) != kernel_source_hash():
-        return None
-    return float(m.group(2))
+    for ln in open(path):
+        cells = [c.strip() for c in ln.strip().strip("|").split("|")]
+        if len(cells) >= 4 and cells[0] == sym and cells[1] == fname:
+            return float(cells[3]) if cells[2] == source_hash(fname) else None
+    return None
 
 
 # ---------------------------------------------------------------- CPU oracle baseline
@@ -440,7 +446,7 @@ def main():
                    "l2": "inputs larger than L2 (Q 134 MB, dO 134 MB, K+V 67 MB, gather tables 5 GB)",
                    "parallelism": f"replicas x{ws}"},
         "pct_of_peak": 100.0 * value / 1e12 / pk["bf16"],
-        "roofline": {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": pk["bf16"],
+        "roofline": {"kernel": f"{dom} ({KERNEL_OF[dom][0]})", "bound": "tensor", "achieved": achieved, "peak": pk["bf16"],
                      "unit": "TFLOP/s", "frac": achieved / pk["bf16"],
                      "frac_of_sustained": achieved / pk["bf16_sustained"],
                      "peak_source": f"{pk['src']} bf16 dense burst", "traffic": tr,

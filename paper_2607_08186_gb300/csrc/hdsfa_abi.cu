@@ -1,12 +1,16 @@
 // C ABI of libhdsfa.so (declared in include/hdsfa.h): host-side validation,
 // problem geometry and kernel dispatch.  No allocation, no synchronisation.
 #include <math.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include "common.cuh"
 
 namespace hdsfa {
 cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L,
                                 int n, int V, int D, int32_t* status, cudaStream_t stream);
+cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
+                              const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
                                const SfaGeom& g, int Dh, float scale, cudaStream_t st);
 cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, float* delta_ws, float* dq_ws,
@@ -53,6 +57,17 @@ hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t m
   return HD_OK;
 }
 
+// HDSFA_KERNELS=mma selects the warp-level mma.sync kernels (the pre-tcgen05
+// baseline, kept for A/B timing); the default is the tcgen05 / TMA path.
+bool use_mma_kernels() {
+  static int v = -1;
+  if (v < 0) {
+    const char* e = getenv("HDSFA_KERNELS");
+    v = (e != nullptr && strcmp(e, "mma") == 0) ? 1 : 0;
+  }
+  return v == 1;
+}
+
 float resolve_scale(float s, int Dh) { return s > 0.f ? s : 1.0f / sqrtf((float)Dh); }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -92,15 +107,14 @@ hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, i
 hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
                     int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode,
                     int window, int32_t* dev_status, cudaStream_t stream) {
-  (void)dev_status;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
     return HD_ERR_INVALID_ARG;
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  return hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream) == cudaSuccess ? HD_OK
-                                                                                       : HD_ERR_CUDA;
+  if (use_mma_kernels()) return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
 }
 
 size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode) {
