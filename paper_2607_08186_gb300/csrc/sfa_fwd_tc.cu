@@ -25,18 +25,17 @@ namespace hdsfa {
 typedef __nv_bfloat16 bf16;
 
 namespace tcfwd {
-constexpr int BM = 128, BN = 128, NST = 2, NTHREADS = 192;
+constexpr int BM = 128, BN = 128, NST = 2, NG = 2, NTHREADS = 64 + NG * 128;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr float kRescaleThreshold = 8.0f;  // log2 units: P stays <= 256 between rescales
+constexpr float kRescaleThreshold = 8.0f;  // log2 units: P stays <= 256 between O rescales
 
 template <int DH>
 struct Smem {
-  bf16 q[BM * DH];        // DH/64 swizzle blocks of [BM][64]
+  bf16 q[NG][BM * DH];  // per query tile: DH/64 swizzle blocks of [BM][64]
   bf16 k[NST][BN * DH];
   bf16 v[NST][BN * DH];
-  bf16 p[BM * BN];        // 2 swizzle blocks of [BM][64]
-  uint64_t q_full, kv_full[NST], kv_empty[NST], s_full[2], s_free[2], p_full, o_done, drain;
+  uint64_t q_full, kv_full[NST], kv_empty[NST], s_full[NG], p_full[NG], o_done[NG], drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -54,20 +53,36 @@ HD_DEVINLINE bool visible(int r, int c, int Lv, int window) {
   return c <= r && c < Lv && (window <= 0 || r - c < window);
 }
 
+// Key-tile range [lo, hi] of the query tile starting at row m0 (hi < lo: no rows).
+HD_DEVINLINE void tile_range(const SfaGeom& G, int m0, int& lo, int& hi) {
+  if (m0 >= G.Lv) {
+    lo = 0;
+    hi = -1;
+    return;
+  }
+  lo = G.window > 0 ? max(0, m0 - G.window + 1) / BN : 0;
+  hi = min(m0 / BN, (G.Lv - 1) / BN);
+}
+
+// TMEM columns: S_g at g*128 (P_g packed bf16 over its first 64 columns), O_g at 256 + g*DH.
 template <int DH>
 __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant__ Params P) {
   extern __shared__ uint8_t smem_raw[];
   Smem<DH>& sm = *reinterpret_cast<Smem<DH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ntile = (G.Lv + BM - 1) / BM;
-  const int mt = ntile - 1 - (int)blockIdx.x;  // longest rows first
-  const int m0 = mt * BM;
+  const int ncta = (G.Lv + NG * BM - 1) / (NG * BM);
+  const int mt = ncta - 1 - (int)blockIdx.x;  // longest rows first
+  const int m0 = mt * NG * BM;
   const int h = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
   const int kvh = h / (G.Hq / G.Hkv);
-  const int n_lo = G.window > 0 ? max(0, m0 - G.window + 1) / BN : 0;
-  const int n_hi = min(mt, (G.Lv - 1) / BN);
-  const int nkv = n_hi - n_lo + 1;
+  int lo[NG], hi[NG];
+#pragma unroll
+  for (int g = 0; g < NG; ++g) tile_range(G, m0 + g * BM, lo[g], hi[g]);
+  const int n_lo = lo[0];
+  int n_hi = hi[0];
+#pragma unroll
+  for (int g = 1; g < NG; ++g) n_hi = max(n_hi, hi[g]);
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.q_full, 1);
@@ -75,12 +90,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
       mbar_init(&sm.kv_full[i], 1);
       mbar_init(&sm.kv_empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.s_full[i], 1);
-      mbar_init(&sm.s_free[i], 128);
+    for (int g = 0; g < NG; ++g) {
+      mbar_init(&sm.s_full[g], 1);
+      mbar_init(&sm.p_full[g], 128);
+      mbar_init(&sm.o_done[g], 1);
     }
-    mbar_init(&sm.p_full, 128);
-    mbar_init(&sm.o_done, 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
     fence_mbar_init();
@@ -101,175 +115,183 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
       tma_prefetch(&P.tm_q);
       tma_prefetch(&P.tm_k);
       tma_prefetch(&P.tm_v);
-      mbar_arrive_expect_tx(&sm.q_full, BM * DH * 2);
-      for (int c = 0; c < DH / 64; ++c)
-        tma_load_5d(sm.q + c * BM * 64, &P.tm_q, &sm.q_full, c * 64, h, s, m0, b);
+      mbar_arrive_expect_tx(&sm.q_full, NG * BM * DH * 2);
+      for (int g = 0; g < NG; ++g)
+        for (int c = 0; c < DH / 64; ++c)
+          tma_load_5d(sm.q[g] + c * BM * 64, &P.tm_q, &sm.q_full, c * 64, h, s, m0 + g * BM, b);
       int issued = 0;
-      for (int it = 0; it < nkv; ++it) {
-        const int st = it % NST;
+      for (int j = n_lo; j <= n_hi; ++j, ++issued) {
+        const int it = j - n_lo, st = it % NST;
         if (it >= NST && !mbar_wait(&sm.kv_empty[st], ((it / NST) - 1) & 1, abort, P.status)) break;
-        const int r0 = (n_lo + it) * BN;
         mbar_arrive_expect_tx(&sm.kv_full[st], 2 * BN * DH * 2);
         for (int c = 0; c < DH / 64; ++c) {
-          tma_load_5d(sm.k[st] + c * BN * 64, &P.tm_k, &sm.kv_full[st], c * 64, kvh, s, r0, b);
-          tma_load_5d(sm.v[st] + c * BN * 64, &P.tm_v, &sm.kv_full[st], c * 64, kvh, s, r0, b);
+          tma_load_5d(sm.k[st] + c * BN * 64, &P.tm_k, &sm.kv_full[st], c * 64, kvh, s, j * BN, b);
+          tma_load_5d(sm.v[st] + c * BN * 64, &P.tm_v, &sm.kv_full[st], c * 64, kvh, s, j * BN, b);
         }
-        ++issued;
       }
-      // let every copy this thread started land before the CTA can exit
+      // every copy this thread started lands before the CTA may exit
       mbar_drain(&sm.q_full, 0);
-      for (int it = max(0, issued - NST); it < issued; ++it)
-        mbar_drain(&sm.kv_full[it % NST], (it / NST) & 1);
+      for (int it = max(0, issued - NST); it < issued; ++it) mbar_drain(&sm.kv_full[it % NST], (it / NST) & 1);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idS = idesc_bf16(BM, BN, 0, 0);  // S[q][kv] = Q K^T, both K-major
-      constexpr uint32_t idO = idesc_bf16(BM, DH, 0, 1);  // O[q][d] += P V, V MN-major
-      const uint32_t qa = smem_u32(sm.q), pa = smem_u32(sm.p);
+      constexpr uint32_t idS = idesc_bf16(BM, BN, 0, 0);  // S[q][kv] = Q K^T (both K-major)
+      constexpr uint32_t idO = idesc_bf16(BM, DH, 0, 1);  // O[q][d] += P V   (P in TMEM, V MN-major)
+      int ps[NG] = {0, 0};                                  // per-group P phases consumed
       bool ok = mbar_wait(&sm.q_full, 0, abort, P.status);
-      auto issue_pv = [&](int jt) -> bool {
-        const int pst = jt % NST;
-        if (!mbar_wait(&sm.p_full, jt & 1, abort, P.status)) return false;
+      int kv_ready = n_lo - 1;                              // highest key tile known loaded
+      auto wait_kv = [&](int j) -> bool {
+        if (j <= kv_ready) return true;
+        const int it = j - n_lo;
+        if (!mbar_wait(&sm.kv_full[it % NST], (it / NST) & 1, abort, P.status)) return false;
+        kv_ready = j;
         tc_fence_after();
-        const uint32_t va = smem_u32(sm.v[pst]);
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(pa + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, BN * 128, 1024);
-          tc_mma_ss(tmem + 256, ad, bd, idO, (jt > 0 || kk > 0) ? 1u : 0u);
-        }
-        tc_commit(&sm.o_done);
-        tc_commit(&sm.kv_empty[pst]);
         return true;
       };
-      for (int it = 0; ok && it < nkv; ++it) {
-        const int st = it % NST, sb = it & 1;
-        if (!mbar_wait(&sm.kv_full[st], (it / NST) & 1, abort, P.status)) break;
-        if (it >= 2 && !mbar_wait(&sm.s_free[sb], ((it - 2) >> 1) & 1, abort, P.status)) break;
-        tc_fence_after();
-        const uint32_t ka = smem_u32(sm.k[st]);
+      auto issue_s = [&](int g, int j) {
+        const uint32_t qa = smem_u32(sm.q[g]), ka = smem_u32(sm.k[(j - n_lo) % NST]);
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
           const uint64_t ad = sdesc_sw128(qa + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
           const uint64_t bd = sdesc_sw128(ka + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
-          tc_mma_ss(tmem + sb * 128, ad, bd, idS, kk > 0 ? 1u : 0u);
+          tc_mma_ss(tmem + g * 128, ad, bd, idS, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&sm.s_full[sb]);
-        if (it >= 1 && !issue_pv(it - 1)) break;
-        if (it == nkv - 1) issue_pv(it);
+        tc_commit(&sm.s_full[g]);
+      };
+      auto issue_pv = [&](int g, int j) -> bool {
+        if (!mbar_wait(&sm.p_full[g], ps[g] & 1, abort, P.status)) return false;
+        ++ps[g];
+        tc_fence_after();
+        const uint32_t va = smem_u32(sm.v[(j - n_lo) % NST]);
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, BN * 128, 1024);
+          tc_mma_ts(tmem + 256 + g * DH, tmem + g * 128 + kk * 8, bd, idO, (j > lo[g] || kk > 0) ? 1u : 0u);
+        }
+        return true;
+      };
+      if (ok && n_hi >= n_lo && wait_kv(n_lo)) {
+        for (int g = 0; g < NG; ++g)
+          if (lo[g] <= n_lo && n_lo <= hi[g]) issue_s(g, n_lo);
+        for (int j = n_lo; ok && j <= n_hi; ++j) {
+          for (int g = 0; ok && g < NG; ++g) {
+            if (lo[g] <= j && j <= hi[g]) {
+              if (!issue_pv(g, j)) { ok = false; break; }
+              if (j == hi[g]) tc_commit(&sm.o_done[g]);
+            }
+            // S of the next tile for this group reuses its S/P columns: issued after its PV
+            if (j + 1 <= hi[g] && lo[g] <= j + 1) {
+              if (!wait_kv(j + 1)) { ok = false; break; }
+              issue_s(g, j + 1);
+            }
+          }
+          tc_commit(&sm.kv_empty[(j - n_lo) % NST]);
+        }
       }
-      // every MMA issued above has finished before TMEM / smem are released
+      // every MMA issued above completes before TMEM / smem are released
       tc_commit(&sm.drain);
       mbar_drain(&sm.drain, 0);
     }
   } else {
     // ------------------------------------------------------------ softmax / epilogue
+    const int g = (warp - 2) >> 2;
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
-    const int r = m0 + row;
+    const int r = m0 + g * BM + row;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
-    float m_run = -INFINITY, l_run = 0.f;
+    const uint32_t tS = tl + g * 128, tO = tl + 256 + g * DH;
+    const float c2 = P.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;  // m_run in raw score units
     bool ok = true;
-    uint8_t* prow = reinterpret_cast<uint8_t*>(sm.p) + row * 128;
-    for (int it = 0; it < nkv; ++it) {
-      const int sb = it & 1;
-      const int j = n_lo + it;
+    for (int j = lo[g]; j <= hi[g]; ++j) {
+      const int i = j - lo[g];
       // tcgen05.ld/st are warp-collective: every wait result is made warp-uniform
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full[sb], (it >> 1) & 1, abort, P.status))) {
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full[g], i & 1, abort, P.status))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      uint32_t sraw[BN];
       float x[BN];
 #pragma unroll
-      for (int c = 0; c < BN / 32; ++c) tmem_ld32(tl + sb * 128 + c * 32, sraw + c * 32);
+      for (int c = 0; c < BN / 32; ++c) tmem_ld32(tS + c * 32, reinterpret_cast<uint32_t*>(x) + c * 32);
       tmem_ld_wait();
-      tc_fence_before();
-      mbar_arrive(&sm.s_free[sb]);
-      const bool need_mask = (j == n_hi) || G.window > 0 || (j + 1) * BN > G.Lv;
-      float tmax = -INFINITY;
+      const bool need_mask = (j == hi[g] && (j + 1) * BN > m0 + g * BM) || G.window > 0 || (j + 1) * BN > G.Lv;
+      if (need_mask) {
 #pragma unroll
-      for (int i = 0; i < BN; ++i) {
-        float y = __uint_as_float(sraw[i]) * P.scale_log2;
-        if (need_mask && !visible(r, j * BN + i, G.Lv, G.window)) y = -INFINITY;
-        x[i] = y;
-        tmax = fmaxf(tmax, y);
+        for (int e = 0; e < BN; ++e)
+          if (!visible(r, j * BN + e, G.Lv, G.window)) x[e] = -INFINITY;
       }
+      float mx[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mx[e] = x[e];
+#pragma unroll
+      for (int e = 8; e < BN; ++e) mx[e & 7] = fmaxf(mx[e & 7], x[e]);
+      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       const float m_new = fmaxf(m_run, tmax);
-      const bool rescale = (m_run == -INFINITY) || (m_new > m_run + kRescaleThreshold);
+      const bool rescale = (m_run == -INFINITY) || ((m_new - m_run) * c2 > kRescaleThreshold);
       const float m_use = rescale ? m_new : m_run;
-      const float m_sub = (m_use == -INFINITY) ? 0.f : m_use;
-      float rsum = 0.f;
+      const float neg = (m_use == -INFINITY) ? 0.f : -m_use * c2;
+      float sum[8];
 #pragma unroll
-      for (int i = 0; i < BN; ++i) {
-        x[i] = exp2f(x[i] - m_sub);
-        rsum += x[i];
+      for (int e = 0; e < 8; ++e) sum[e] = 0.f;
+      uint32_t pk[BN / 2];
+#pragma unroll
+      for (int e = 0; e < BN; e += 2) {
+        const float p0 = ex2_approx(fmaf(x[e], c2, neg));
+        const float p1 = ex2_approx(fmaf(x[e + 1], c2, neg));
+        sum[(e >> 1) & 7] += p0 + p1;
+        pk[e >> 1] = cvt_bf16x2(p0, p1);
       }
-      if (it > 0) {
-        // PV of the previous tile must be done: it reads the P buffer and writes O
-        if (!__all_sync(0xffffffffu, mbar_wait(&sm.o_done, (it - 1) & 1, abort, P.status))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const bool mine = rescale && m_run != -INFINITY;
-        if (__any_sync(0xffffffffu, mine)) {
-          const float alpha = mine ? exp2f(m_run - m_use) : 1.f;
-          l_run *= alpha;
+      const float rsum = ((sum[0] + sum[1]) + (sum[2] + sum[3])) + ((sum[4] + sum[5]) + (sum[6] + sum[7]));
+      // O_g already holds every earlier tile's PV (its S of this tile was issued after them)
+      const bool mine = rescale && m_run != -INFINITY && i > 0;
+      if (__any_sync(0xffffffffu, mine)) {
+        const float alpha = mine ? ex2_approx((m_run - m_use) * c2) : 1.f;
+        l_run *= alpha;
 #pragma unroll
-          for (int c = 0; c < DH / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(tl + 256 + c * 32, o);
-            tmem_ld_wait();
+        for (int c = 0; c < DH / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-            tmem_st32(tl + 256 + c * 32, o);
-          }
-          tmem_st_wait();
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          tmem_st32(tO + c * 32, o);
         }
       }
       m_run = m_use;
       l_run += rsum;
-      // P row -> shared memory, 128-byte swizzle, two 64-column blocks
+      // P (bf16 pairs) over the first 64 columns of this group's S
 #pragma unroll
-      for (int c = 0; c < BN / 8; ++c) {
-        uint4 w;
-        w.x = pack_bf16(x[c * 8 + 0], x[c * 8 + 1]);
-        w.y = pack_bf16(x[c * 8 + 2], x[c * 8 + 3]);
-        w.z = pack_bf16(x[c * 8 + 4], x[c * 8 + 5]);
-        w.w = pack_bf16(x[c * 8 + 6], x[c * 8 + 7]);
-        const int blk = c >> 3, ch = (c & 7) ^ (row & 7);
-        *reinterpret_cast<uint4*>(prow + blk * (BM * 128) + ch * 16) = w;
-      }
-      fence_async_smem();
+      for (int c = 0; c < BN / 32; ++c) tmem_st16(tS + c * 16, pk + c * 16);
+      tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&sm.p_full);
+      mbar_arrive(&sm.p_full[g]);
     }
-    if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.o_done, (nkv - 1) & 1, abort, P.status))) {
+    if (ok && hi[g] >= lo[g] && __all_sync(0xffffffffu, mbar_wait(&sm.o_done[g], 0, abort, P.status))) {
       tc_fence_after();
       const float inv = 1.f / l_run;
       bf16* orow = P.o + (((long long)b * G.nL + (long long)r * G.rs + s) * G.Hq + h) * DH;
 #pragma unroll
       for (int c = 0; c < DH / 32; ++c) {
         uint32_t o[32];
-        tmem_ld32(tl + 256 + c * 32, o);
+        tmem_ld32(tO + c * 32, o);
         tmem_ld_wait();
         if (r < G.Lv) {
 #pragma unroll
           for (int e = 0; e < 32; e += 8) {
             uint4 w;
-            w.x = pack_bf16(__uint_as_float(o[e + 0]) * inv, __uint_as_float(o[e + 1]) * inv);
-            w.y = pack_bf16(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
-            w.z = pack_bf16(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv);
-            w.w = pack_bf16(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv);
+            w.x = cvt_bf16x2(__uint_as_float(o[e + 0]) * inv, __uint_as_float(o[e + 1]) * inv);
+            w.y = cvt_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
+            w.z = cvt_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv);
+            w.w = cvt_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv);
             *reinterpret_cast<uint4*>(orow + c * 32 + e) = w;
           }
         }
       }
       if (r < G.Lv)
-        P.lse[((long long)b * G.Hq + h) * G.nL + (long long)r * G.rs + s] = (m_run + log2f(l_run)) * kLn2;
+        P.lse[((long long)b * G.Hq + h) * G.nL + (long long)r * G.rs + s] = (m_run * c2 + log2f(l_run)) * kLn2;
     }
   }
 
@@ -320,7 +342,7 @@ static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   const int smem = (int)sizeof(tcfwd::Smem<DH>) + 1024;
   cudaError_t e = cudaFuncSetAttribute(tcfwd::fwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((p.g.Lv + tcfwd::BM - 1) / tcfwd::BM, p.g.Hq * p.g.ns, p.g.B);
+  dim3 grid((p.g.Lv + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM), p.g.Hq * p.g.ns, p.g.B);
   tcfwd::fwd_kernel<DH><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }
