@@ -198,10 +198,10 @@ class HotPath:
         b.sfa_fwd(self.q, self.k, self.v, self.o, self.lse, s.n, self.mode)
         if ev is not None:
             ev[1].record()
-        b.sfa_bwd_prep(self.o, self.do, s.n, self.mode, self.ws, s.Hkv)
+        b.sfa_bwd_prep(self.o, self.do, self.lse, s.n, self.mode, self.ws, s.Hkv)
         if ev is not None:
             ev[2].record()
-        b.sfa_bwd_main(self.q, self.k, self.v, self.lse, self.do, self.dk, self.dv, s.n, self.mode, self.ws)
+        b.sfa_bwd_main(self.q, self.k, self.v, self.do, self.dk, self.dv, s.n, self.mode, self.ws)
         if ev is not None:
             ev[3].record()
         b.sfa_bwd_finalize(self.dq, s.n, self.mode, self.ws, s.Hkv)
@@ -265,10 +265,11 @@ def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2):
 # ABI phase -> (kernel symbol, source file) of the implementation the library runs.
 KERNEL_OF = {
     "sfa_fwd": ("hdsfa::tcfwd::fwd_kernel<128>", "sfa_fwd_tc.cu"),
-    "sfa_bwd_main": ("hdsfa::sfa_bwd_mma_kernel<128>", "sfa_mma.cu"),
+    "sfa_bwd_main": ("hdsfa::tcbwd::bwd_kernel", "sfa_bwd_tc.cu"),
 }
 if os.environ.get("HDSFA_KERNELS") == "mma":
     KERNEL_OF["sfa_fwd"] = ("hdsfa::sfa_fwd_mma_kernel<128>", "sfa_mma.cu")
+    KERNEL_OF["sfa_bwd_main"] = ("hdsfa::sfa_bwd_mma_kernel<128>", "sfa_mma.cu")
 
 
 def source_hash(fname: str) -> str:

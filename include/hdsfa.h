@@ -78,8 +78,9 @@ hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float*
                     int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode,
                     int window, int32_t* dev_status, cudaStream_t stream);
 
-/* Bytes of device workspace sfa_bwd needs for these sizes (fp32 dQ accumulator
- * [B][nL][Hq][Dh] plus fp32 row terms [B][Hq][nL]).  Returns 0 for invalid sizes. */
+/* Bytes of device workspace sfa_bwd needs for these sizes and mode (fp32 dQ
+ * accumulator [B][nL][Hq][Dh] plus two fp32 row terms of about B*Hq*nL each).
+ * Returns 0 for invalid sizes. */
 size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode);
 
 /*
@@ -101,20 +102,21 @@ hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, 
 
 /*
  * The three phases sfa_bwd runs, in order on one stream, exported so a caller
- * can overlap or time them separately.  Same arguments and workspace as sfa_bwd.
- *   sfa_bwd_prep     : delta[b][h][p] = sum_d dO*O (fp32) into the workspace and
- *                      zero the workspace's fp32 dQ accumulator.
- *   sfa_bwd_main     : recompute P, accumulate dQ (fp32, workspace) and write dk, dv.
+ * can overlap or time them separately.  Same sizes, mode and workspace as sfa_bwd.
+ *   sfa_bwd_prep     : delta = rowsum(dO * O) and lse * log2(e) into the workspace
+ *                      (fp32, stream-major), and zero its fp32 dQ accumulator.
+ *   sfa_bwd_main     : recompute P on visible pairs, add every dQ contribution
+ *                      into the accumulator and write dk, dv (overwritten).
  *   sfa_bwd_finalize : dq = bf16(scale * accumulator).
  * A later phase reads what the earlier one left in the workspace.
  */
-hd_status_t sfa_bwd_prep(const void* o, const void* dout, int B, int L, int n, int Hq, int Hkv,
-                         int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
+hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int B, int L, int n, int Hq,
+                         int Hkv, int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
                          cudaStream_t stream);
-hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const float* lse,
-                         const void* dout, void* dk, void* dv, int B, int L, int n, int Hq, int Hkv,
-                         int Dh, float softmax_scale, sfa_mode_t mode, int window, void* workspace,
-                         size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream);
+hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void* dout, void* dk, void* dv,
+                         int B, int L, int n, int Hq, int Hkv, int Dh, float softmax_scale,
+                         sfa_mode_t mode, int window, void* workspace, size_t workspace_bytes,
+                         int32_t* dev_status, cudaStream_t stream);
 hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
                              float softmax_scale, sfa_mode_t mode, void* workspace,
                              size_t workspace_bytes, cudaStream_t stream);

@@ -50,9 +50,9 @@ def lib():
             L.sfa_bwd.restype = I
             L.sfa_bwd.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
             L.sfa_bwd_prep.restype = I
-            L.sfa_bwd_prep.argtypes = [P, P, I, I, I, I, I, I, I, P, Z, P]
+            L.sfa_bwd_prep.argtypes = [P, P, P, I, I, I, I, I, I, I, P, Z, P]
             L.sfa_bwd_main.restype = I
-            L.sfa_bwd_main.argtypes = [P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
+            L.sfa_bwd_main.argtypes = [P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
             L.sfa_bwd_finalize.restype = I
             L.sfa_bwd_finalize.argtypes = [P, I, I, I, I, I, I, F, I, P, Z, P]
             L.hd_status_string.restype = ctypes.c_char_p
@@ -126,19 +126,19 @@ def _wsb(ws):
     return ws.numel() * ws.element_size()
 
 
-def sfa_bwd_prep(o, dout, n, mode, workspace, Hkv, stream=None):
-    """Phase 1 of sfa_bwd: delta = rowsum(dO * O) and a zeroed dQ accumulator (workspace)."""
+def sfa_bwd_prep(o, dout, lse, n, mode, workspace, Hkv, stream=None):
+    """Phase 1 of sfa_bwd: delta = rowsum(dO * O), lse * log2(e), zeroed dQ accumulator."""
     B, nL, Hq, Dh = o.shape
-    _check(lib().sfa_bwd_prep(_p(o), _p(dout), B, nL // n, n, Hq, Hkv, Dh, int(mode), _p(workspace),
-                              _wsb(workspace), _stream(stream)), "sfa_bwd_prep")
+    _check(lib().sfa_bwd_prep(_p(o), _p(dout), _p(lse), B, nL // n, n, Hq, Hkv, Dh, int(mode),
+                              _p(workspace), _wsb(workspace), _stream(stream)), "sfa_bwd_prep")
 
 
-def sfa_bwd_main(q, k, v, lse, dout, dk, dv, n, mode, workspace, softmax_scale=0.0, window=0,
+def sfa_bwd_main(q, k, v, dout, dk, dv, n, mode, workspace, softmax_scale=0.0, window=0,
                  dev_status=None, stream=None):
     """Phase 2 of sfa_bwd: dK, dV and the fp32 dQ accumulator."""
     B, L, Hq, Hkv, Dh = _attn_dims(q, k, n)
-    _check(lib().sfa_bwd_main(_p(q), _p(k), _p(v), _p(lse), _p(dout), _p(dk), _p(dv), B, L, n, Hq,
-                              Hkv, Dh, float(softmax_scale), int(mode), int(window), _p(workspace),
+    _check(lib().sfa_bwd_main(_p(q), _p(k), _p(v), _p(dout), _p(dk), _p(dv), B, L, n, Hq, Hkv, Dh,
+                              float(softmax_scale), int(mode), int(window), _p(workspace),
                               _wsb(workspace), _p(dev_status), _stream(stream)), "sfa_bwd_main")
 
 

@@ -13,12 +13,16 @@ cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void*
                               const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
                                const SfaGeom& g, int Dh, float scale, cudaStream_t st);
-cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, float* delta_ws, float* dq_ws,
-                                const SfaGeom& g, int Dh, cudaStream_t st);
-cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const float* lse,
-                                    const void* dout, void* dk, void* dv, const float* delta_ws,
+cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
+                                float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
+                                cudaStream_t st);
+cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const void* dout,
+                                    void* dk, void* dv, const float* lse2_ws, const float* delta_ws,
                                     float* dq_ws, const SfaGeom& g, int Dh, float scale,
                                     cudaStream_t st);
+cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, const void* dout, void* dk,
+                                   void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
+                                   const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
                                     float scale, cudaStream_t st);
 }  // namespace hdsfa
@@ -72,19 +76,31 @@ float resolve_scale(float s, int Dh) { return s > 0.f ? s : 1.0f / sqrtf((float)
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then fp32 delta [B][Hq][nL].
+// Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then lse*log2(e) and
+// delta, each fp32 [B][Hq][ns][Lvp] (stream-major rows, Lvp = Lv rounded up to 64).
 struct BwdWs {
   float* dq;
+  float* lse2;
   float* delta;
 };
 
-hd_status_t split_ws(const SfaGeom& g, int Dh, void* ws, size_t bytes, BwdWs* out) {
+size_t ws_bytes(const SfaGeom& g, int Dh) {
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
-  const size_t need = align256(rows * Dh * sizeof(float)) + align256(rows * sizeof(float));
-  if (ws == nullptr || bytes < need || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+  const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)((g.Lv + 63) & ~63);
+  return align256(rows * Dh * sizeof(float)) + 2 * align256(trows * sizeof(float));
+}
+
+hd_status_t split_ws(const SfaGeom& g, int Dh, void* ws, size_t bytes, BwdWs* out) {
+  if (ws == nullptr || bytes < ws_bytes(g, Dh) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
     return HD_ERR_WORKSPACE;
-  out->dq = static_cast<float*>(ws);
-  out->delta = reinterpret_cast<float*>(static_cast<char*>(ws) + align256(rows * Dh * sizeof(float)));
+  const size_t rows = (size_t)g.B * g.nL * g.Hq;
+  const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)((g.Lv + 63) & ~63);
+  char* p = static_cast<char*>(ws);
+  out->dq = reinterpret_cast<float*>(p);
+  p += align256(rows * Dh * sizeof(float));
+  out->lse2 = reinterpret_cast<float*>(p);
+  p += align256(trows * sizeof(float));
+  out->delta = reinterpret_cast<float*>(p);
   return HD_OK;
 }
 
@@ -120,37 +136,40 @@ hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float*
 size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode) {
   SfaGeom g;
   if (make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g) != HD_OK) return 0;
-  const size_t rows = (size_t)B * g.nL * Hq;
-  return align256(rows * Dh * sizeof(float)) + align256(rows * sizeof(float));
+  return ws_bytes(g, Dh);
 }
 
-hd_status_t sfa_bwd_prep(const void* o, const void* dout, int B, int L, int n, int Hq, int Hkv,
-                         int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
+hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int B, int L, int n, int Hq,
+                         int Hkv, int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
                          cudaStream_t stream) {
-  if (!aligned16(o) || !aligned16(dout)) return HD_ERR_INVALID_ARG;
+  if (!aligned16(o) || !aligned16(dout) || !aligned16(lse)) return HD_ERR_INVALID_ARG;
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
   if (st != HD_OK) return st;
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
-  return cuda_status(hdsfa::launch_sfa_bwd_prep(o, dout, ws.delta, ws.dq, g, Dh, stream));
+  return cuda_status(hdsfa::launch_sfa_bwd_prep(o, dout, lse, ws.lse2, ws.delta, ws.dq, g, Dh, stream));
 }
 
-hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const float* lse,
-                         const void* dout, void* dk, void* dv, int B, int L, int n, int Hq, int Hkv,
-                         int Dh, float softmax_scale, sfa_mode_t mode, int window, void* workspace,
-                         size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream) {
-  (void)dev_status;
-  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(lse) || !aligned16(dout) ||
-      !aligned16(dk) || !aligned16(dv))
+hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void* dout, void* dk, void* dv,
+                         int B, int L, int n, int Hq, int Hkv, int Dh, float softmax_scale,
+                         sfa_mode_t mode, int window, void* workspace, size_t workspace_bytes,
+                         int32_t* dev_status, cudaStream_t stream) {
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dout) || !aligned16(dk) ||
+      !aligned16(dv))
     return HD_ERR_INVALID_ARG;
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
-  return cuda_status(hdsfa::launch_sfa_bwd_main_mma(q, k, v, lse, dout, dk, dv, ws.delta, ws.dq, g,
-                                                    Dh, resolve_scale(softmax_scale, Dh), stream));
+  const float scale = resolve_scale(softmax_scale, Dh);
+  // head dim 128 runs on the tcgen05 kernel; head dim 64 on the mma.sync kernel
+  if (Dh == 128 && !use_mma_kernels())
+    return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
+                                                     scale, dev_status, stream));
+  return cuda_status(hdsfa::launch_sfa_bwd_main_mma(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh,
+                                                    scale, stream));
 }
 
 hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
@@ -179,10 +198,10 @@ hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, 
   if (st != HD_OK) return st;
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
-  st = sfa_bwd_prep(o, dout, B, L, n, Hq, Hkv, Dh, mode, workspace, workspace_bytes, stream);
+  st = sfa_bwd_prep(o, dout, lse, B, L, n, Hq, Hkv, Dh, mode, workspace, workspace_bytes, stream);
   if (st != HD_OK) return st;
-  st = sfa_bwd_main(q, k, v, lse, dout, dk, dv, B, L, n, Hq, Hkv, Dh, softmax_scale, mode, window,
-                    workspace, workspace_bytes, dev_status, stream);
+  st = sfa_bwd_main(q, k, v, dout, dk, dv, B, L, n, Hq, Hkv, Dh, softmax_scale, mode, window, workspace,
+                    workspace_bytes, dev_status, stream);
   if (st != HD_OK) return st;
   return sfa_bwd_finalize(dq, B, L, n, Hq, Hkv, Dh, softmax_scale, mode, workspace,
                           workspace_bytes, stream);

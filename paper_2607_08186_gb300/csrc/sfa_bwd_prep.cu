@@ -1,0 +1,102 @@
+// Backward pre- and post-processing (bandwidth kernels).
+//
+// prep:     delta[p] = sum_d dO[p,d] * O[p,d] (fp32) and lse2[p] = lse[p] * log2(e),
+//           both written stream-major, [B][Hq][ns][Lvp] with row r of stream s at
+//           position p = r*ns + s and Lvp = Lv rounded up to 64, so one query tile
+//           of any stream is 64 contiguous floats (a single bulk copy).  Rows in
+//           [Lv, Lvp) get lse2 = +inf and delta = 0 (their P and dS vanish).
+//           Also zeroes the fp32 dQ accumulator.
+// finalize: dq = bf16(scale * accumulator), round to nearest even.
+#include "common.cuh"
+
+namespace hdsfa {
+
+typedef __nv_bfloat16 bf16;
+
+template <int DH>
+__global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restrict__ o,
+                                                           const bf16* __restrict__ dout,
+                                                           const float* __restrict__ lse,
+                                                           float* __restrict__ lse2_t,
+                                                           float* __restrict__ delta_t,
+                                                           float* __restrict__ dq_acc, SfaGeom g) {
+  const int lane = threadIdx.x & 31;
+  const long long row = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // (b, p, h)
+  if (row >= (long long)g.B * g.nL * g.Hq) return;
+  float acc = 0.f;
+  if (lane < DH / 8) {
+    const uint4 x = *reinterpret_cast<const uint4*>(o + row * DH + lane * 8);
+    const uint4 y = *reinterpret_cast<const uint4*>(dout + row * DH + lane * 8);
+    const bf16* xa = reinterpret_cast<const bf16*>(&x);
+    const bf16* ya = reinterpret_cast<const bf16*>(&y);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc += __bfloat162float(xa[i]) * __bfloat162float(ya[i]);
+  }
+#pragma unroll
+  for (int off = 16; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  float4* dqr = reinterpret_cast<float4*>(dq_acc + row * DH);
+  for (int c = lane; c < DH / 4; c += 32) dqr[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (lane == 0) {
+    const long long h = row % g.Hq, bp = row / g.Hq, p = bp % g.nL, b = bp / g.nL;
+    const int Lvp = (g.Lv + 63) & ~63;
+    const long long s = p % g.ns, r = p / g.ns;
+    const long long t = ((b * g.Hq + h) * g.ns + s) * Lvp + r;
+    delta_t[t] = acc;
+    lse2_t[t] = lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
+  }
+}
+
+__global__ void sfa_bwd_pad_kernel(float* __restrict__ lse2_t, float* __restrict__ delta_t, SfaGeom g) {
+  const int Lvp = (g.Lv + 63) & ~63, pad = Lvp - g.Lv;
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (long long)g.B * g.Hq * g.ns * pad) return;
+  const long long t = (i / pad) * Lvp + g.Lv + i % pad;
+  lse2_t[t] = INFINITY;
+  delta_t[t] = 0.f;
+}
+
+__global__ void __launch_bounds__(256) sfa_bwd_finalize_kernel(const float* __restrict__ dq_acc,
+                                                               bf16* __restrict__ dq, long long n8,
+                                                               float scale) {
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n8) return;
+  const float4 a = reinterpret_cast<const float4*>(dq_acc)[2 * i];
+  const float4 c = reinterpret_cast<const float4*>(dq_acc)[2 * i + 1];
+  uint4 r;
+  r.x = pack_bf16(a.x * scale, a.y * scale);
+  r.y = pack_bf16(a.z * scale, a.w * scale);
+  r.z = pack_bf16(c.x * scale, c.y * scale);
+  r.w = pack_bf16(c.z * scale, c.w * scale);
+  reinterpret_cast<uint4*>(dq)[i] = r;
+}
+
+cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
+                                float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
+                                cudaStream_t st) {
+  const long long rows = (long long)g.B * g.nL * g.Hq;
+  const unsigned blocks = (unsigned)((rows * 32 + 255) / 256);
+  if (Dh == 64)
+    sfa_bwd_prep_kernel<64><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, lse, lse2_ws,
+                                                   delta_ws, dq_ws, g);
+  else
+    sfa_bwd_prep_kernel<128><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, lse, lse2_ws,
+                                                    delta_ws, dq_ws, g);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int pad = ((g.Lv + 63) & ~63) - g.Lv;
+  if (pad > 0) {
+    const long long n = (long long)g.B * g.Hq * g.ns * pad;
+    sfa_bwd_pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(lse2_ws, delta_ws, g);
+    e = cudaGetLastError();
+  }
+  return e;
+}
+
+cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
+                                    float scale, cudaStream_t st) {
+  const long long n8 = (long long)g.B * g.nL * g.Hq * Dh / 8;
+  sfa_bwd_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dq_ws, (bf16*)dq, n8, scale);
+  return cudaGetLastError();
+}
+
+}  // namespace hdsfa

@@ -16,8 +16,6 @@
 //               only when the running max grows by more than 2^8, epilogue.
 // Shared-memory tiles use the 128-byte swizzle written by TMA; P is written by
 // the softmax threads in the same layout.  Every mbarrier wait is bounded.
-#include <cudaTypedefs.h>
-
 #include "tc_common.cuh"
 
 namespace hdsfa {
@@ -306,37 +304,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
 }  // namespace tcfwd
 
 // --------------------------------------------------------------------- host
-static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (fn == nullptr) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
-  return fn;
-}
-
-// Tensor map over a [B][nL][H][Dh] bf16 tensor seen as the 5-D array
-// {Dh, H, ns, Lv, B} (innermost first): virtual row r of stream s is position
-// r*rs + s.  Box = 64 head-dim elements (one 128-byte swizzle row) x box_rows rows.
-bool make_rows_tmap(CUtensorMap* m, const void* base, const SfaGeom& g, int H, int Dh, int box_rows) {
-  auto enc = tmap_encoder();
-  if (enc == nullptr) return false;
-  const cuuint64_t e = 2;
-  cuuint64_t dims[5] = {(cuuint64_t)Dh, (cuuint64_t)H, (cuuint64_t)g.ns, (cuuint64_t)g.Lv, (cuuint64_t)g.B};
-  cuuint64_t strides[4] = {Dh * e, (cuuint64_t)H * Dh * e, (cuuint64_t)g.rs * H * Dh * e,
-                           (cuuint64_t)g.nL * H * Dh * e};
-  cuuint32_t box[5] = {64, 1, 1, (cuuint32_t)box_rows, 1};
-  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS;
-}
-
 template <int DH>
 static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   const int smem = (int)sizeof(tcfwd::Smem<DH>) + 1024;

@@ -32,8 +32,8 @@ struct MmaBwdArgs {
   const bf16* k;
   const bf16* v;
   const bf16* dout;
-  const float* lse;
-  const float* delta;  // [B][Hq][nL] rowsum(dO * O)
+  const float* lse2;   // [B][Hq][ns][Lvp] lse * log2(e), stream-major (see sfa_bwd_prep.cu)
+  const float* delta;  // [B][Hq][ns][Lvp] rowsum(dO * O)
   float* dq_acc;       // [B][nL][Hq][Dh] fp32, pre-zeroed; gets sum dS K (unscaled)
   bf16* dk;
   bf16* dv;
@@ -221,51 +221,6 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
 }
 
 // ----------------------------------------------------------------- backward
-// delta[b][h][p] = sum_d dO * O (fp32), and zero the fp32 dQ accumulator row.
-template <int DH>
-__global__ void __launch_bounds__(256) sfa_bwd_pre_kernel(const bf16* __restrict__ o,
-                                                          const bf16* __restrict__ dout,
-                                                          float* __restrict__ delta,
-                                                          float* __restrict__ dq_acc, int B,
-                                                          int nL, int Hq) {
-  const int lane = threadIdx.x & 31;
-  const long long row = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // (b, p, h)
-  if (row >= (long long)B * nL * Hq) return;
-  float acc = 0.f;
-  if (lane < DH / 8) {
-    const uint4 x = *reinterpret_cast<const uint4*>(o + row * DH + lane * 8);
-    const uint4 y = *reinterpret_cast<const uint4*>(dout + row * DH + lane * 8);
-    const bf16* xa = reinterpret_cast<const bf16*>(&x);
-    const bf16* ya = reinterpret_cast<const bf16*>(&y);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) acc += __bfloat162float(xa[i]) * __bfloat162float(ya[i]);
-  }
-#pragma unroll
-  for (int off = 16; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  float4* dqr = reinterpret_cast<float4*>(dq_acc + row * DH);
-  for (int c = lane; c < DH / 4; c += 32) dqr[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (lane == 0) {
-    const long long h = row % Hq, bp = row / Hq, p = bp % nL, b = bp / nL;
-    delta[(b * Hq + h) * nL + p] = acc;
-  }
-}
-
-// dq = scale * dq_acc, fp32 -> bf16 (round to nearest even), 8 elements per thread.
-__global__ void __launch_bounds__(256) sfa_bwd_post_kernel(const float* __restrict__ dq_acc,
-                                                           bf16* __restrict__ dq, long long n8,
-                                                           float scale) {
-  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n8) return;
-  const float4 a = reinterpret_cast<const float4*>(dq_acc)[2 * i];
-  const float4 c = reinterpret_cast<const float4*>(dq_acc)[2 * i + 1];
-  uint4 r;
-  r.x = pack_bf16(a.x * scale, a.y * scale);
-  r.y = pack_bf16(a.z * scale, a.w * scale);
-  r.z = pack_bf16(c.x * scale, c.y * scale);
-  r.w = pack_bf16(c.z * scale, c.w * scale);
-  reinterpret_cast<uint4*>(dq)[i] = r;
-}
-
 // One CTA per (key tile j, b, K/V head g, stream s).  It keeps dK_j, dV_j in
 // registers while looping over the group's query heads and the query tiles that
 // can see tile j; dQ contributions go to the fp32 accumulator with atomics.
@@ -300,11 +255,12 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   auto q_base = [&](const bf16* t, int h) {
     return t + (((long long)b * G.nL + s) * G.Hq + h) * DH;
   };
+  const int Lvp = (G.Lv + 63) & ~63;
   auto row_terms = [&](int it, int r, float& l2, float& dl) {
     const int h = kvh * grp + it / nq, m0 = (j + it % nq) * BM;
-    const long long idx = ((long long)b * G.Hq + h) * G.nL + (long long)(m0 + r) * G.rs + s;
+    const long long idx = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + m0 + r;
     const bool ok = m0 + r < G.Lv;
-    l2 = ok ? a.lse[idx] * kLog2e : 0.f;
+    l2 = ok ? a.lse2[idx] : 0.f;
     dl = ok ? a.delta[idx] : 0.f;
   };
 
@@ -506,24 +462,11 @@ cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void
   return Dh == 64 ? fwd_impl<64>(a, st) : fwd_impl<128>(a, st);
 }
 
-cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, float* delta_ws, float* dq_ws,
-                                const SfaGeom& g, int Dh, cudaStream_t st) {
-  const long long rows = (long long)g.B * g.nL * g.Hq;
-  const unsigned blocks = (unsigned)((rows * 32 + 255) / 256);
-  if (Dh == 64)
-    sfa_bwd_pre_kernel<64><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, delta_ws,
-                                                  dq_ws, g.B, g.nL, g.Hq);
-  else
-    sfa_bwd_pre_kernel<128><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, delta_ws,
-                                                   dq_ws, g.B, g.nL, g.Hq);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const float* lse,
-                                    const void* dout, void* dk, void* dv, const float* delta_ws,
+cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const void* dout,
+                                    void* dk, void* dv, const float* lse2_ws, const float* delta_ws,
                                     float* dq_ws, const SfaGeom& g, int Dh, float scale,
                                     cudaStream_t st) {
-  MmaBwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)dout, lse, delta_ws,
+  MmaBwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)dout, lse2_ws, delta_ws,
                dq_ws, (bf16*)dk, (bf16*)dv, g, scale, scale * kLog2e};
   dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.ns, g.B);
   auto smem_of = [](int dh) {
@@ -541,13 +484,6 @@ cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v,
     if (e != cudaSuccess) return e;
     sfa_bwd_mma_kernel<128><<<grid, NT, smem, st>>>(a);
   }
-  return cudaGetLastError();
-}
-
-cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
-                                    float scale, cudaStream_t st) {
-  const long long n8 = (long long)g.B * g.nL * g.Hq * Dh / 8;
-  sfa_bwd_post_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dq_ws, (bf16*)dq, n8, scale);
   return cudaGetLastError();
 }
 

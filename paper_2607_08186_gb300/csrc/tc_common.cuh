@@ -76,6 +76,29 @@ HD_DEVINLINE void tma_load_5d(void* dst, const CUtensorMap* m, uint64_t* bar, in
       : "memory");
 }
 
+// 1-D bulk copy global -> shared (16-byte aligned, size a multiple of 16).
+HD_DEVINLINE void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Tiled reduce-add shared -> global through a tensor map (fp32 add); elements
+// outside the tensor are skipped.  Tracked by the issuing thread's bulk group.
+HD_DEVINLINE void tma_reduce_add_5d(const CUtensorMap* m, const void* src, int c0, int c1, int c2, int c3,
+                                    int c4) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.5d.global.shared::cta.add.tile.bulk_group"
+      " [%0, {%2, %3, %4, %5, %6}], [%1];\n" ::"l"(reinterpret_cast<uint64_t>(m)),
+      "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+      : "memory");
+}
+HD_DEVINLINE void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
+HD_DEVINLINE void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+HD_DEVINLINE void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
+
 // ---------------------------------------------------------------- tcgen05
 HD_DEVINLINE void tmem_alloc(uint32_t* dst, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(dst)),
@@ -186,5 +209,13 @@ HD_DEVINLINE void tmem_st32(uint32_t taddr, const uint32_t* r) {
 }
 HD_DEVINLINE void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 HD_DEVINLINE void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
+
+// ---------------------------------------------------------------- host: tensor maps
+// Tensor map over a [B][nL][H][Dh] tensor (element size esize) seen as the 5-D array
+// {Dh, H, ns, Lv, B} (innermost first): virtual row r of stream s is position
+// r*rs + s.  Box = box_d elements x box_rows rows; swizzle128 selects the
+// 128-byte swizzle (box_d * esize must then be 128).  Defined in tmap.cu.
+bool make_rows_tmap(CUtensorMap* m, const void* base, const SfaGeom& g, int H, int Dh, int box_rows,
+                    int esize = 2, int box_d = 64, bool swizzle128 = true);
 
 }  // namespace hdsfa

@@ -19,25 +19,36 @@ TOL_LSE = 1e-3
 TOL_GRAD = 1e-2
 
 
-def gpu_fwd(q, k, v, n, mode, scale=0.0, window=0):
+def check_status(st):
+    """The device status word must stay clear (no bounded wait expired, no bad index)."""
+    torch.cuda.synchronize()
+    v = int(st.item())
+    assert v == 0, f"device status bits set: {v:#x}"
+
+
+def gpu_fwd(q, k, v, n, mode, scale=0.0, window=0, status=None):
     qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
     B, nL, Hq, Dh = q.shape
     o = torch.empty_like(qd)
     lse = torch.empty(B, Hq, nL, dtype=torch.float32, device="cuda")
-    binding.sfa_fwd(qd, kd, vd, o, lse, n, mode, scale or 0.0, window)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda") if status is None else status
+    binding.sfa_fwd(qd, kd, vd, o, lse, n, mode, scale or 0.0, window, dev_status=st)
+    if status is None:
+        check_status(st)
     return qd, kd, vd, o, lse
 
 
 def gpu_fwd_bwd(q, k, v, do, n, mode, scale=0.0, window=0):
-    qd, kd, vd, o, lse = gpu_fwd(q, k, v, n, mode, scale, window)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    qd, kd, vd, o, lse = gpu_fwd(q, k, v, n, mode, scale, window, status=st)
     dod = do.cuda()
     B, nL, Hq, Dh = q.shape
     Hkv = k.shape[2]
     dq, dk, dv = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
     wsb = binding.sfa_bwd_workspace_bytes(B, nL // n, n, Hq, Hkv, Dh, mode)
     ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
-    binding.sfa_bwd(qd, kd, vd, o, lse, dod, dq, dk, dv, n, mode, ws, scale or 0.0, window)
-    torch.cuda.synchronize()
+    binding.sfa_bwd(qd, kd, vd, o, lse, dod, dq, dk, dv, n, mode, ws, scale or 0.0, window, dev_status=st)
+    check_status(st)
     return o.cpu(), lse.cpu(), dq.cpu(), dk.cpu(), dv.cpu()
 
 
