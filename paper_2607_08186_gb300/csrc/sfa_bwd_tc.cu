@@ -6,20 +6,26 @@
 // tiles that can see tile j (causal: query tiles at or after the key tile; LOCAL:
 // also within the window).  Per query tile, with TMEM lane = key row:
 //   S^T  = K Q^T,  dP^T = V dO^T                      (SS MMA, M=128 N=64 K=128)
-//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)   (softmax WG)
+//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)   (softmax)
 //   dV  += P^T dO,  dK += dS^T Q                      (TS MMA: P^T, dS^T bf16 in TMEM)
 //   dQ^T = K^T dS^T                                   (SS MMA, M=128 (head dim) N=64)
 // dQ^T leaves TMEM through the dQ warpgroup: shared memory, then a TMA tensor
 // reduce-add (fp32) into the workspace accumulator.  dK, dV stay in TMEM for
 // the whole loop and are written once (dK scaled).
 //
-// Roles (320 threads): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer,
-// warps 2..5 softmax (one key row each), warps 6..9 dQ flush (one head-dim row
-// each).  Q/dO/lse2/delta tiles and the S^T/dP^T/dQ^T TMEM buffers are
-// double-buffered; every mbarrier wait is bounded.
+// Issue order of the MMA thread for tile t:
+//   dP(t+1) | wait P(t) | dV(t) S(t+1) dK(t) | wait dQ^T read-out of t-1 | dQ(t)
+// so the softmax of tile t+1 (which needs S(t+1), dP(t+1)) runs while the tensor
+// pipe works on dK(t), dQ(t) and dP(t+2).  S(t+1) reuses the S^T columns that hold
+// P^T(t) only after dV(t) has been issued (tcgen05 MMAs of one thread run in order).
 //
-// TMEM columns: S^T[st] at 64*st (P^T bf16 over its first 32), dP^T[st] at
-// 128 + 64*st (dS^T bf16 over its first 32, then dQ^T fp32), dV at 256, dK at 384.
+// Roles (448 threads): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer,
+// warps 2..5 and 6..9 softmax (key row = TMEM lane; query columns 0..31 and
+// 32..63), warps 10..13 dQ flush (one head-dim row each).  Every mbarrier wait
+// is bounded.
+//
+// TMEM columns: S^T at 0 (P^T bf16 over its first 32), dP^T[st] at 64 + 64*st
+// (dS^T bf16 over its first 32), dQ^T at 192, dV at 256, dK at 384.
 #include "tc_common.cuh"
 
 namespace hdsfa {
@@ -27,10 +33,9 @@ namespace hdsfa {
 typedef __nv_bfloat16 bf16;
 
 namespace tcbwd {
-constexpr int BK = 128, BQ = 64, DH = 128, NST = 2, NTHREADS = 320;
-constexpr uint32_t COL_DV = 256, COL_DK = 384;
-HD_DEVINLINE uint32_t col_st(int st) { return 64u * st; }
-HD_DEVINLINE uint32_t col_dpt(int st) { return 128u + 64u * st; }
+constexpr int BK = 128, BQ = 64, DH = 128, NST = 2, NTHREADS = 448;
+constexpr uint32_t COL_ST = 0, COL_DQ = 192, COL_DV = 256, COL_DK = 384;
+HD_DEVINLINE uint32_t col_dpt(int st) { return 64u + 64u * st; }
 
 struct Smem {
   bf16 k[BK * DH];          // 2 swizzle blocks of [128 key rows][64]
@@ -41,8 +46,8 @@ struct Smem {
   float dq[4][BQ * 32];     // per dQ warp: [64 queries][32 head-dim] fp32 staging
   float lse2[NST][BQ];
   float delta[NST][BQ];
-  uint64_t kv_full, qd_full[NST], qd_empty[NST], sdp_full[NST], p_ready[NST], dq_full[NST], dq_free[NST],
-      kv_done, drain;
+  uint64_t kv_full, qd_full[NST], qd_empty[NST], s_full, dp_full[NST], p_ready, dq_full, dq_free,
+      ds_free[NST], s_read, kv_done, drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -83,11 +88,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     for (int i = 0; i < NST; ++i) {
       mbar_init(&sm.qd_full[i], 1);
       mbar_init(&sm.qd_empty[i], 1);
-      mbar_init(&sm.sdp_full[i], 1);
-      mbar_init(&sm.p_ready[i], 128);
-      mbar_init(&sm.dq_full[i], 1);
-      mbar_init(&sm.dq_free[i], 128);
+      mbar_init(&sm.dp_full[i], 1);
+      mbar_init(&sm.ds_free[i], 1);
     }
+    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.p_ready, 256);
+    mbar_init(&sm.s_read, 256);
+    mbar_init(&sm.dq_full, 1);
+    mbar_init(&sm.dq_free, 128);
     mbar_init(&sm.kv_done, 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
@@ -139,143 +147,159 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       constexpr uint32_t idKV = idesc_bf16(128, DH, 0, 1);  // dV, dK: A in TMEM, B = dO/Q MN-major
       constexpr uint32_t idQ = idesc_bf16(128, BQ, 1, 1);   // dQ^T: A = K^T, B = dS^T, both MN-major
       const uint32_t ka = smem_u32(sm.k), va = smem_u32(sm.v);
-      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status);
-      auto issue_rest = [&](int u) -> bool {
-        const int su = u & 1;
-        if (!mbar_wait(&sm.p_ready[su], (u >> 1) & 1, abort, P.status)) return false;
+      // S^T = K Q^T or dP^T = V dO^T of tile t into TMEM column col
+      auto issue_sdp = [&](uint32_t aa, const bf16* bt, uint32_t col) {
+        const uint32_t ba = smem_u32(bt);
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint64_t ad = sdesc_sw128(aa + (kk >> 2) * (BK * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = sdesc_sw128(ba + (kk >> 2) * (BQ * 128) + (kk & 3) * 32, 16, 1024);
+          tc_mma_ss(tmem + col, ad, bd, idS, kk > 0 ? 1u : 0u);
+        }
+      };
+      // dV (a_col = P^T) or dK (a_col = dS^T) += A * B, B = dO or Q of the tile (MN-major)
+      auto issue_kv = [&](uint32_t a_col, const bf16* bt, uint32_t d_col, bool acc) {
+        const uint32_t ba = smem_u32(bt);
+#pragma unroll
+        for (int kk = 0; kk < BQ / 16; ++kk) {
+          const uint64_t bd = sdesc_sw128(ba + kk * 16 * 128, BQ * 128, 1024);
+          tc_mma_ts(tmem + d_col, tmem + a_col + kk * 8, bd, idKV, (acc || kk > 0) ? 1u : 0u);
+        }
+      };
+      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.qd_full[0], 0, abort, P.status);
+      if (ok) {
         tc_fence_after();
-        const uint32_t qa = smem_u32(sm.q[su]), da = smem_u32(sm.dO[su]), dsa = smem_u32(sm.ds[su]);
-#pragma unroll
-        for (int kk = 0; kk < BQ / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(da + kk * 16 * 128, BQ * 128, 1024);
-          tc_mma_ts(tmem + COL_DV, tmem + col_st(su) + kk * 8, bd, idKV, (u > 0 || kk > 0) ? 1u : 0u);
+        issue_sdp(ka, sm.q[0], COL_ST);
+        tc_commit(&sm.s_full);
+        issue_sdp(va, sm.dO[0], col_dpt(0));
+        tc_commit(&sm.dp_full[0]);
+      }
+      for (int t = 0; ok && t < T; ++t) {
+        const int st = t & 1, sn = st ^ 1;
+        if (t + 1 < T) {
+          // dP^T(t+1): its columns last held dS^T(t-1), read by dK(t-1) issued earlier
+          if (!mbar_wait(&sm.qd_full[sn], ((t + 1) >> 1) & 1, abort, P.status)) { ok = false; break; }
+          tc_fence_after();
+          issue_sdp(va, sm.dO[sn], col_dpt(sn));
+          tc_commit(&sm.dp_full[sn]);
         }
-#pragma unroll
-        for (int kk = 0; kk < BQ / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(qa + kk * 16 * 128, BQ * 128, 1024);
-          tc_mma_ts(tmem + COL_DK, tmem + col_dpt(su) + kk * 8, bd, idKV, (u > 0 || kk > 0) ? 1u : 0u);
+        if (!mbar_wait(&sm.p_ready, t & 1, abort, P.status)) { ok = false; break; }
+        tc_fence_after();
+        issue_kv(COL_ST, sm.dO[st], COL_DV, t > 0);
+        if (t + 1 < T) {
+          issue_sdp(ka, sm.q[sn], COL_ST);  // after dV(t) read P^T(t)
+          tc_commit(&sm.s_full);
         }
-        tc_commit(&sm.qd_empty[su]);
-        // dQ^T overwrites the dP^T / dS^T columns only after the dK MMA above read them
+        issue_kv(col_dpt(st), sm.q[st], COL_DK, t > 0);
+        tc_commit(&sm.qd_empty[st]);
+        if (t >= 1 && !mbar_wait(&sm.dq_free, (t - 1) & 1, abort, P.status)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t dsa = smem_u32(sm.ds[st]);
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
           const uint64_t ad = sdesc_sw128(ka + kk * 16 * 128, BK * 128, 1024);
           const uint64_t bd = sdesc_sw128(dsa + kk * 16 * 128, BK * 128, 1024);
-          tc_mma_ss(tmem + col_dpt(su), ad, bd, idQ, kk > 0 ? 1u : 0u);
+          tc_mma_ss(tmem + COL_DQ, ad, bd, idQ, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&sm.dq_full[su]);
-        return true;
-      };
-      for (int t = 0; ok && t < T; ++t) {
-        const int st = t & 1;
-        if (!mbar_wait(&sm.qd_full[st], (t >> 1) & 1, abort, P.status)) break;
-        if (t >= NST && !mbar_wait(&sm.dq_free[st], ((t - NST) >> 1) & 1, abort, P.status)) break;
-        tc_fence_after();
-        const uint32_t qa = smem_u32(sm.q[st]), da = smem_u32(sm.dO[st]);
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint64_t ak = sdesc_sw128(ka + (kk >> 2) * (BK * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bq = sdesc_sw128(qa + (kk >> 2) * (BQ * 128) + (kk & 3) * 32, 16, 1024);
-          tc_mma_ss(tmem + col_st(st), ak, bq, idS, kk > 0 ? 1u : 0u);
-        }
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint64_t av = sdesc_sw128(va + (kk >> 2) * (BK * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bo = sdesc_sw128(da + (kk >> 2) * (BQ * 128) + (kk & 3) * 32, 16, 1024);
-          tc_mma_ss(tmem + col_dpt(st), av, bo, idS, kk > 0 ? 1u : 0u);
-        }
-        tc_commit(&sm.sdp_full[st]);
-        if (t >= 1 && !issue_rest(t - 1)) { ok = false; break; }
+        tc_commit(&sm.dq_full);
+        tc_commit(&sm.ds_free[st]);
       }
-      if (ok && T > 0) ok = issue_rest(T - 1);
       tc_commit(&sm.kv_done);
       tc_commit(&sm.drain);
       mbar_drain(&sm.drain, 0);
     }
-  } else if (warp < 6) {
+  } else if (warp < 10) {
     // ------------------------------------------------------------ softmax (key rows)
+    const int half = (warp - 2) >> 2;  // query columns [32*half, 32*half + 32)
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
     const int kr = n0 + row;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     const float c2 = P.scale_log2;
-    uint8_t* dsrow0 = reinterpret_cast<uint8_t*>(sm.ds[0]) + row * 128;
-    uint8_t* dsrow1 = reinterpret_cast<uint8_t*>(sm.ds[1]) + row * 128;
     bool ok = true;
     for (int t = 0; t < T; ++t) {
       const int st = t & 1;
-      const int q0 = (i_lo + t % nq) * BQ;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.sdp_full[st], (t >> 1) & 1, abort, P.status))) {
+      const int q0 = (i_lo + t % nq) * BQ + 32 * half;
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status) &&
+                                       mbar_wait(&sm.dp_full[st], (t >> 1) & 1, abort, P.status))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      uint32_t sr[BQ], dr[BQ];
-      tmem_ld32(tl + col_st(st), sr);
-      tmem_ld32(tl + col_st(st) + 32, sr + 32);
-      tmem_ld32(tl + col_dpt(st), dr);
-      tmem_ld32(tl + col_dpt(st) + 32, dr + 32);
+      uint32_t sr[32], dr[32];
+      tmem_ld32(tl + COL_ST + 32 * half, sr);
+      tmem_ld32(tl + col_dpt(st) + 32 * half, dr);
       tmem_ld_wait();
-      const float* l2 = sm.lse2[st];
-      const float* dl = sm.delta[st];
-      const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + BQ > G.Lv);
-      uint32_t pp[BQ / 2], dd[BQ / 2];
-#pragma unroll
-      for (int c = 0; c < BQ; c += 2) {
-        float p0 = ex2_approx(fmaf(__uint_as_float(sr[c]), c2, -l2[c]));
-        float p1 = ex2_approx(fmaf(__uint_as_float(sr[c + 1]), c2, -l2[c + 1]));
-        if (need_mask) {
-          if (!visible(q0 + c, kr, G.Lv, G.window)) p0 = 0.f;
-          if (!visible(q0 + c + 1, kr, G.Lv, G.window)) p1 = 0.f;
-        }
-        const float d0 = p0 * (__uint_as_float(dr[c]) - dl[c]);
-        const float d1 = p1 * (__uint_as_float(dr[c + 1]) - dl[c + 1]);
-        pp[c >> 1] = cvt_bf16x2(p0, p1);
-        dd[c >> 1] = cvt_bf16x2(d0, d1);
-      }
-      tmem_st16(tl + col_st(st), pp);
-      tmem_st16(tl + col_st(st) + 16, pp + 16);
-      tmem_st16(tl + col_dpt(st), dd);
-      tmem_st16(tl + col_dpt(st) + 16, dd + 16);
-      // dS^T row -> shared memory for the dQ MMA; the buffer was last read by tile t-2's dQ MMA
-      if (t >= NST && !__all_sync(0xffffffffu, mbar_wait(&sm.dq_full[st], ((t - NST) >> 1) & 1, abort, P.status))) {
+      // both halves have read their S^T / dP^T columns before either packs bf16 over them
+      // (an mbarrier rather than bar.sync, so an aborted peer cannot strand this warp)
+      tc_fence_before();
+      mbar_arrive(&sm.s_read);
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_read, t & 1, abort, P.status))) {
         ok = false;
         break;
       }
-      uint8_t* dsrow = st ? dsrow1 : dsrow0;
+      tc_fence_after();
+      const float4* l2 = reinterpret_cast<const float4*>(sm.lse2[st] + 32 * half);
+      const float4* dl = reinterpret_cast<const float4*>(sm.delta[st] + 32 * half);
+      const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + 32 > G.Lv);
+      uint32_t pp[16], dd[16];
 #pragma unroll
-      for (int c = 0; c < 8; ++c)
-        *reinterpret_cast<uint4*>(dsrow + ((c ^ (row & 7)) << 4)) =
+      for (int c4 = 0; c4 < 8; ++c4) {
+        const float4 lv = l2[c4], dv = dl[c4];
+        const float la[4] = {lv.x, lv.y, lv.z, lv.w}, da[4] = {dv.x, dv.y, dv.z, dv.w};
+        float p[4], d[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int c = c4 * 4 + e;
+          p[e] = ex2_approx(fmaf(__uint_as_float(sr[c]), c2, -la[e]));
+          if (need_mask && !visible(q0 + c, kr, G.Lv, G.window)) p[e] = 0.f;
+          d[e] = p[e] * (__uint_as_float(dr[c]) - da[e]);
+        }
+        pp[2 * c4] = cvt_bf16x2(p[0], p[1]);
+        pp[2 * c4 + 1] = cvt_bf16x2(p[2], p[3]);
+        dd[2 * c4] = cvt_bf16x2(d[0], d[1]);
+        dd[2 * c4 + 1] = cvt_bf16x2(d[2], d[3]);
+      }
+      // P^T and dS^T (bf16 pairs) over the first 32 columns of S^T and dP^T[st]
+      tmem_st16(tl + COL_ST + 16 * half, pp);
+      tmem_st16(tl + col_dpt(st) + 16 * half, dd);
+      // dS^T -> shared memory for the dQ MMA; this buffer was last read by dQ(t-2)
+      if (t >= NST &&
+          !__all_sync(0xffffffffu, mbar_wait(&sm.ds_free[st], ((t - NST) >> 1) & 1, abort, P.status))) {
+        ok = false;
+        break;
+      }
+      uint8_t* dsrow = reinterpret_cast<uint8_t*>(sm.ds[st]) + row * 128;
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        *reinterpret_cast<uint4*>(dsrow + (((4 * half + c) ^ (row & 7)) << 4)) =
             make_uint4(dd[4 * c], dd[4 * c + 1], dd[4 * c + 2], dd[4 * c + 3]);
       fence_async_smem();
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&sm.p_ready[st]);
+      mbar_arrive(&sm.p_ready);
     }
-    // dK, dV epilogue: this thread's key row
+    // epilogue: half 0 writes this key row of dV, half 1 of dK (scaled)
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
       tc_fence_after();
       const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + s) * G.Hkv + kvh) * DH;
+      const float mul = half ? P.scale : 1.f;
+      bf16* dst = (half ? P.dk : P.dv) + orow;
+      const uint32_t col = half ? COL_DK : COL_DV;
 #pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        const float mul = which ? P.scale : 1.f;
-        bf16* dst = (which ? P.dk : P.dv) + orow;
-        const uint32_t col = which ? COL_DK : COL_DV;
+      for (int c = 0; c < DH / 32; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tl + col + c * 32, o);
+        tmem_ld_wait();
+        if (kr < G.Lv) {
 #pragma unroll
-        for (int c = 0; c < DH / 32; ++c) {
-          uint32_t o[32];
-          tmem_ld32(tl + col + c * 32, o);
-          tmem_ld_wait();
-          if (kr < G.Lv) {
-#pragma unroll
-            for (int e = 0; e < 32; e += 8) {
-              uint4 w;
-              w.x = cvt_bf16x2(__uint_as_float(o[e + 0]) * mul, __uint_as_float(o[e + 1]) * mul);
-              w.y = cvt_bf16x2(__uint_as_float(o[e + 2]) * mul, __uint_as_float(o[e + 3]) * mul);
-              w.z = cvt_bf16x2(__uint_as_float(o[e + 4]) * mul, __uint_as_float(o[e + 5]) * mul);
-              w.w = cvt_bf16x2(__uint_as_float(o[e + 6]) * mul, __uint_as_float(o[e + 7]) * mul);
-              *reinterpret_cast<uint4*>(dst + c * 32 + e) = w;
-            }
+          for (int e = 0; e < 32; e += 8) {
+            uint4 w;
+            w.x = cvt_bf16x2(__uint_as_float(o[e + 0]) * mul, __uint_as_float(o[e + 1]) * mul);
+            w.y = cvt_bf16x2(__uint_as_float(o[e + 2]) * mul, __uint_as_float(o[e + 3]) * mul);
+            w.z = cvt_bf16x2(__uint_as_float(o[e + 4]) * mul, __uint_as_float(o[e + 5]) * mul);
+            w.w = cvt_bf16x2(__uint_as_float(o[e + 6]) * mul, __uint_as_float(o[e + 7]) * mul);
+            *reinterpret_cast<uint4*>(dst + c * 32 + e) = w;
           }
         }
       }
@@ -286,16 +310,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     float* stage = sm.dq[q4];
     for (int t = 0; t < T; ++t) {
-      const int st = t & 1;
       const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full[st], (t >> 1) & 1, abort, P.status))) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) break;
       tc_fence_after();
       uint32_t v[BQ];
-      tmem_ld32(tl + col_dpt(st), v);
-      tmem_ld32(tl + col_dpt(st) + 32, v + 32);
+      tmem_ld32(tl + COL_DQ, v);
+      tmem_ld32(tl + COL_DQ + 32, v + 32);
       tmem_ld_wait();
       tc_fence_before();
-      mbar_arrive(&sm.dq_free[st]);
+      mbar_arrive(&sm.dq_free);
       // the previous reduce must have finished reading the staging buffer
       if (lane == 0) bulk_wait_read0();
       __syncwarp();

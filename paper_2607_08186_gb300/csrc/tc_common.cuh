@@ -62,6 +62,11 @@ HD_DEVINLINE void mbar_drain(uint64_t* bar, uint32_t parity) {
   }
 }
 
+// Barrier among `nthreads` threads (whole warps) of the CTA on hardware barrier `id` (1..15).
+HD_DEVINLINE void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
+}
+
 // ---------------------------------------------------------------- TMA
 HD_DEVINLINE void tma_prefetch(const CUtensorMap* m) {
   asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
