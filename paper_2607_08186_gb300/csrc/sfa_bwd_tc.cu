@@ -242,6 +242,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       const float4* l2 = reinterpret_cast<const float4*>(sm.lse2[st] + 32 * half);
       const float4* dl = reinterpret_cast<const float4*>(sm.delta[st] + 32 * half);
       const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + 32 > G.Lv);
+      if (need_mask) {
+        // zero the scores of invisible pairs up front: exp2(-inf) = 0 below
+#pragma unroll
+        for (int c = 0; c < 32; ++c)
+          if (!visible(q0 + c, kr, G.Lv, G.window)) sr[c] = __float_as_uint(-INFINITY);
+      }
       uint32_t pp[16], dd[16];
 #pragma unroll
       for (int c4 = 0; c4 < 8; ++c4) {
@@ -252,7 +258,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         for (int e = 0; e < 4; ++e) {
           const int c = c4 * 4 + e;
           p[e] = ex2_approx(fmaf(__uint_as_float(sr[c]), c2, -la[e]));
-          if (need_mask && !visible(q0 + c, kr, G.Lv, G.window)) p[e] = 0.f;
           d[e] = p[e] * (__uint_as_float(dr[c]) - da[e]);
         }
         pp[2 * c4] = cvt_bf16x2(p[0], p[1]);
