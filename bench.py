@@ -273,8 +273,12 @@ if os.environ.get("HDSFA_KERNELS") == "mma":
 
 
 def source_hash(fname: str) -> str:
-    with open(os.path.join(ROOT, "paper_2607_08186_gb300", "csrc", fname), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """sha256 prefix of a kernel's source file plus the device headers it includes."""
+    h = hashlib.sha256()
+    for part in (fname, "tc_common.cuh", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2607_08186_gb300", "csrc", part), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def traffic_record(phase: str):

@@ -14,19 +14,18 @@
 // the whole loop and are written once (dK scaled).
 //
 // Issue order of the MMA thread for tile t:
-//   S(t+1) | wait dQ^T(t-1) read-out | dP(t+1) | wait P(t) | dV(t) dK(t) dQ(t)
-// so the softmax of tile t+1 runs while the tensor pipe works on dV(t), dK(t),
-// dQ(t).  S^T and dP^T are double-buffered by tile parity; dQ^T(t) reuses the dP^T
-// columns of tile t once dK(t) (issued before it, and tcgen05 MMAs of one thread
-// run in order) has read dS^T from them.
+//   dP(t+1) | wait P(t) | dV(t) S(t+1) dK(t) | wait dQ^T read-out of t-1 | dQ(t)
+// so the softmax of tile t+1 (which needs S(t+1), dP(t+1)) runs while the tensor
+// pipe works on dK(t), dQ(t) and dP(t+2).  S(t+1) reuses the S^T columns that hold
+// P^T(t) only after dV(t) has been issued (tcgen05 MMAs of one thread run in order).
 //
 // Roles (448 threads): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer,
 // warps 2..5 and 6..9 softmax (key row = TMEM lane; query columns 0..31 and
 // 32..63), warps 10..13 dQ flush (one head-dim row each).  Every mbarrier wait
 // is bounded.
 //
-// TMEM columns: S^T[st] at 64*st (P^T bf16 over its first 32), dP^T[st] at
-// 128 + 64*st (dS^T bf16 over its first 32, then dQ^T fp32), dV at 256, dK at 384.
+// TMEM columns: S^T at 0 (P^T bf16 over its first 32), dP^T[st] at 64 + 64*st
+// (dS^T bf16 over its first 32), dQ^T at 192, dV at 256, dK at 384.
 #include "tc_common.cuh"
 
 namespace hdsfa {
@@ -35,9 +34,8 @@ typedef __nv_bfloat16 bf16;
 
 namespace tcbwd {
 constexpr int BK = 128, BQ = 64, DH = 128, NST = 2, NTHREADS = 448;
-constexpr uint32_t COL_DV = 256, COL_DK = 384;
-HD_DEVINLINE uint32_t col_st(int st) { return 64u * st; }
-HD_DEVINLINE uint32_t col_dpt(int st) { return 128u + 64u * st; }
+constexpr uint32_t COL_ST = 0, COL_DQ = 192, COL_DV = 256, COL_DK = 384;
+HD_DEVINLINE uint32_t col_dpt(int st) { return 64u + 64u * st; }
 
 struct Smem {
   bf16 k[BK * DH];          // 2 swizzle blocks of [128 key rows][64]
@@ -48,8 +46,8 @@ struct Smem {
   float dq[4][BQ * 32];     // per dQ warp: [64 queries][32 head-dim] fp32 staging
   float lse2[NST][BQ];
   float delta[NST][BQ];
-  uint64_t kv_full, qd_full[NST], qd_empty[NST], s_full[NST], dp_full[NST], p_ready[NST], dq_full[NST],
-      dq_free[NST], s_read, kv_done, drain;
+  uint64_t kv_full, qd_full[NST], qd_empty[NST], s_full, dp_full[NST], p_ready, dq_full, dq_free,
+      ds_free[NST], s_read, kv_done, drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -91,12 +89,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       mbar_init(&sm.qd_full[i], 1);
       mbar_init(&sm.qd_empty[i], 1);
       mbar_init(&sm.dp_full[i], 1);
-      mbar_init(&sm.s_full[i], 1);
-      mbar_init(&sm.p_ready[i], 256);
-      mbar_init(&sm.dq_full[i], 1);
-      mbar_init(&sm.dq_free[i], 128);
+      mbar_init(&sm.ds_free[i], 1);
     }
+    mbar_init(&sm.s_full, 1);
+    mbar_init(&sm.p_ready, 256);
     mbar_init(&sm.s_read, 256);
+    mbar_init(&sm.dq_full, 1);
+    mbar_init(&sm.dq_free, 128);
     mbar_init(&sm.kv_done, 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
@@ -170,39 +169,40 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.qd_full[0], 0, abort, P.status);
       if (ok) {
         tc_fence_after();
-        issue_sdp(ka, sm.q[0], col_st(0));
-        tc_commit(&sm.s_full[0]);
+        issue_sdp(ka, sm.q[0], COL_ST);
+        tc_commit(&sm.s_full);
         issue_sdp(va, sm.dO[0], col_dpt(0));
         tc_commit(&sm.dp_full[0]);
       }
       for (int t = 0; ok && t < T; ++t) {
         const int st = t & 1, sn = st ^ 1;
         if (t + 1 < T) {
-          // S^T(t+1): its columns last held P^T(t-1), read by dV(t-1) issued earlier
+          // dP^T(t+1): its columns last held dS^T(t-1), read by dK(t-1) issued earlier
           if (!mbar_wait(&sm.qd_full[sn], ((t + 1) >> 1) & 1, abort, P.status)) { ok = false; break; }
-          tc_fence_after();
-          issue_sdp(ka, sm.q[sn], col_st(sn));
-          tc_commit(&sm.s_full[sn]);
-          // dP^T(t+1): its columns last held dQ^T(t-1), which must have been read out
-          if (t >= 1 && !mbar_wait(&sm.dq_free[sn], ((t - 1) >> 1) & 1, abort, P.status)) { ok = false; break; }
           tc_fence_after();
           issue_sdp(va, sm.dO[sn], col_dpt(sn));
           tc_commit(&sm.dp_full[sn]);
         }
-        if (!mbar_wait(&sm.p_ready[st], (t >> 1) & 1, abort, P.status)) { ok = false; break; }
+        if (!mbar_wait(&sm.p_ready, t & 1, abort, P.status)) { ok = false; break; }
         tc_fence_after();
-        issue_kv(col_st(st), sm.dO[st], COL_DV, t > 0);
+        issue_kv(COL_ST, sm.dO[st], COL_DV, t > 0);
+        if (t + 1 < T) {
+          issue_sdp(ka, sm.q[sn], COL_ST);  // after dV(t) read P^T(t)
+          tc_commit(&sm.s_full);
+        }
         issue_kv(col_dpt(st), sm.q[st], COL_DK, t > 0);
         tc_commit(&sm.qd_empty[st]);
-        // dQ^T(t) over dP^T(t) / dS^T(t), after dK(t) read dS^T
+        if (t >= 1 && !mbar_wait(&sm.dq_free, (t - 1) & 1, abort, P.status)) { ok = false; break; }
+        tc_fence_after();
         const uint32_t dsa = smem_u32(sm.ds[st]);
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
           const uint64_t ad = sdesc_sw128(ka + kk * 16 * 128, BK * 128, 1024);
           const uint64_t bd = sdesc_sw128(dsa + kk * 16 * 128, BK * 128, 1024);
-          tc_mma_ss(tmem + col_dpt(st), ad, bd, idQ, kk > 0 ? 1u : 0u);
+          tc_mma_ss(tmem + COL_DQ, ad, bd, idQ, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&sm.dq_full[st]);
+        tc_commit(&sm.dq_full);
+        tc_commit(&sm.ds_free[st]);
       }
       tc_commit(&sm.kv_done);
       tc_commit(&sm.drain);
@@ -220,14 +220,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     for (int t = 0; t < T; ++t) {
       const int st = t & 1;
       const int q0 = (i_lo + t % nq) * BQ + 32 * half;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full[st], (t >> 1) & 1, abort, P.status) &&
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status) &&
                                        mbar_wait(&sm.dp_full[st], (t >> 1) & 1, abort, P.status))) {
         ok = false;
         break;
       }
       tc_fence_after();
       uint32_t sr[32], dr[32];
-      tmem_ld32(tl + col_st(st) + 32 * half, sr);
+      tmem_ld32(tl + COL_ST + 32 * half, sr);
       tmem_ld32(tl + col_dpt(st) + 32 * half, dr);
       tmem_ld_wait();
       // both halves have read their S^T / dP^T columns before either packs bf16 over them
@@ -266,11 +266,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         dd[2 * c4 + 1] = cvt_bf16x2(d[2], d[3]);
       }
       // P^T and dS^T (bf16 pairs) over the first 32 columns of S^T and dP^T[st]
-      tmem_st16(tl + col_st(st) + 16 * half, pp);
+      tmem_st16(tl + COL_ST + 16 * half, pp);
       tmem_st16(tl + col_dpt(st) + 16 * half, dd);
       // dS^T -> shared memory for the dQ MMA; this buffer was last read by dQ(t-2)
       if (t >= NST &&
-          !__all_sync(0xffffffffu, mbar_wait(&sm.dq_full[st], ((t - NST) >> 1) & 1, abort, P.status))) {
+          !__all_sync(0xffffffffu, mbar_wait(&sm.ds_free[st], ((t - NST) >> 1) & 1, abort, P.status))) {
         ok = false;
         break;
       }
@@ -282,7 +282,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       fence_async_smem();
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&sm.p_ready[st]);
+      mbar_arrive(&sm.p_ready);
     }
     // epilogue: half 0 writes this key row of dV, half 1 of dK (scaled)
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
@@ -316,15 +316,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     float* stage = sm.dq[q4];
     for (int t = 0; t < T; ++t) {
       const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
-      const int st = t & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full[st], (t >> 1) & 1, abort, P.status))) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) break;
       tc_fence_after();
       uint32_t v[BQ];
-      tmem_ld32(tl + col_dpt(st), v);
-      tmem_ld32(tl + col_dpt(st) + 32, v + 32);
+      tmem_ld32(tl + COL_DQ, v);
+      tmem_ld32(tl + COL_DQ + 32, v + 32);
       tmem_ld_wait();
       tc_fence_before();
-      mbar_arrive(&sm.dq_free[st]);
+      mbar_arrive(&sm.dq_free);
       // the previous reduce must have finished reading the staging buffer
       if (lane == 0) bulk_wait_read0();
       __syncwarp();
