@@ -2,30 +2,35 @@
 // head dim 128.
 //
 // One CTA owns a 128-row key tile j of one virtual causal problem (SfaGeom) and
-// one K/V head; it loops over the group's query heads and over the 64-row query
+// one K/V head; it loops over the group's query heads and over the 128-row query
 // tiles that can see tile j (causal: query tiles at or after the key tile; LOCAL:
-// also within the window).  Per query tile, with TMEM lane = key row:
-//   S^T  = K Q^T,  dP^T = V dO^T                      (SS MMA, M=128 N=64 K=128)
-//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)   (softmax)
-//   dV  += P^T dO,  dK += dS^T Q                      (TS MMA: P^T, dS^T bf16 in TMEM)
-//   dQ^T = K^T dS^T                                   (SS MMA, M=128 (head dim) N=64)
-// dQ^T leaves TMEM through the dQ warpgroup: shared memory, then a TMA tensor
-// reduce-add (fp32) into the workspace accumulator.  dK, dV stay in TMEM for
-// the whole loop and are written once (dK scaled).
+// also within the window).  Every GEMM is a 128 x 128 x 16k tcgen05 MMA (N = 128
+// runs at full tensor rate; N = 64 does not):
+//   S^T  = K Q^T,  dP^T = V dO^T        SS: A = K / V (K-major), B = Q / dO (K-major)
+//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)      (softmax)
+//   dV  += P^T dO,  dK += dS^T Q        TS: A = P^T / dS^T packed bf16 in TMEM
+//   dQ   = dS K                         SS: A = dS^T tile in smem read MN-major,
+//                                           B = K read MN-major; TMEM lane = query row
+// dK and dV stay in TMEM for the whole loop and are written once (dK scaled).  dQ
+// of each tile is read out by the dQ warpgroup, staged in shared
+// memory (128-byte swizzle) and added into the fp32 workspace accumulator by TMA
+// tensor reduce-add.
 //
-// Issue order of the MMA thread for tile t:
-//   dP(t+1) | wait P(t) | dV(t) S(t+1) dK(t) | wait dQ^T read-out of t-1 | dQ(t)
-// so the softmax of tile t+1 (which needs S(t+1), dP(t+1)) runs while the tensor
-// pipe works on dK(t), dQ(t) and dP(t+2).  S(t+1) reuses the S^T columns that hold
-// P^T(t) only after dV(t) has been issued (tcgen05 MMAs of one thread run in order).
+// TMEM: two 128-column regions R0, R1 swap roles with the tile parity p:
+//   S^T(t) in R[p] (P^T packed bf16 over its first 64 columns, then dQ(t)),
+//   dP^T(t) in R[p^1] (dS^T packed bf16 over its first 64 columns);  dV at 256, dK at 384.
+// MMA issue order:  wait P(t) | dV(t) dK(t) dQ(t) | S(t+1) | wait dQ(t) read-out | dP(t+1)
+// S(t+1) lands in R[p^1], whose dS^T(t) dK(t) has already consumed (tcgen05 MMAs of
+// one thread execute in order), so it overlaps the dQ(t) read-out; dP(t+1) lands in
+// R[p] only after that read-out.
 //
-// Roles (448 threads): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer,
-// warps 2..5 and 6..9 softmax (key row = TMEM lane; query columns 0..31 and
-// 32..63), warps 10..13 dQ flush (one head-dim row each).  Every mbarrier wait
-// is bounded.
-//
-// TMEM columns: S^T at 0 (P^T bf16 over its first 32), dP^T[st] at 64 + 64*st
-// (dS^T bf16 over its first 32), dQ^T at 192, dV at 256, dK at 384.
+// Roles (448 threads, at most 4 warps per scheduler so each thread keeps 128
+// registers): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer, warps 2..5
+// softmax (TMEM lane = key row; 128 query columns in four 32-column chunks),
+// warps 6..9 / 10..13 dQ flush for head-dim columns 0..63 / 64..127 (TMEM lane =
+// query row): each loads its 64 columns, releases the TMEM, then stages two 4 KB
+// rounds through its own buffer.
+// Every mbarrier wait is bounded.
 #include "tc_common.cuh"
 
 namespace hdsfa {
@@ -33,24 +38,27 @@ namespace hdsfa {
 typedef __nv_bfloat16 bf16;
 
 namespace tcbwd {
-constexpr int BK = 128, BQ = 64, DH = 128, NST = 2, NTHREADS = 448;
-constexpr uint32_t COL_ST = 0, COL_DQ = 192, COL_DV = 256, COL_DK = 384;
-HD_DEVINLINE uint32_t col_dpt(int st) { return 64u + 64u * st; }
+constexpr int BK = 128, BQ = 128, DH = 128, NTHREADS = 448;
+constexpr uint32_t COL_DV = 256, COL_DK = 384;
+HD_DEVINLINE uint32_t col_r(int r) { return 128u * r; }
 
 struct Smem {
-  bf16 k[BK * DH];          // 2 swizzle blocks of [128 key rows][64]
+  bf16 k[BK * DH];        // 2 swizzle blocks of [128 key rows][64]
   bf16 v[BK * DH];
-  bf16 q[NST][BQ * DH];     // 2 swizzle blocks of [64 query rows][64]
-  bf16 dO[NST][BQ * DH];
-  bf16 ds[NST][BK * BQ];    // dS^T [128 key rows][64 queries], one swizzle block
-  float dq[4][BQ * 32];     // per dQ warp: [64 queries][32 head-dim] fp32 staging
-  float lse2[NST][BQ];
-  float delta[NST][BQ];
-  uint64_t kv_full, qd_full[NST], qd_empty[NST], s_full, dp_full[NST], p_ready, dq_full, dq_free,
-      ds_free[NST], s_read, kv_done, drain;
+  bf16 q[2][BQ * DH];     // double-buffered query tile: 2 swizzle blocks of [128 rows][64]
+  bf16 dO[BQ * DH];
+  bf16 ds[BK * BQ];       // dS^T [128 key rows][128 queries]: 2 swizzle blocks of [128][64]
+  float dqs[8][32 * 32];  // per dQ warp: [32 query rows][32 head-dim] fp32, 128-byte swizzle
+  float lse2[BQ];
+  float delta[BQ];
+  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, p_ready, dq_full, dq_free,
+      kv_done, drain;
   uint32_t tmem_base;
   int abort;
 };
+
+// dynamic shared memory (plus the 1 KB alignment pad) must fit the 227 KB per-block limit
+static_assert(sizeof(Smem) + 1024 <= 232448, "backward shared-memory layout exceeds 227 KB");
 
 struct Params {
   CUtensorMap tm_q, tm_do, tm_k, tm_v, tm_dq;
@@ -85,17 +93,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.kv_full, 1);
-    for (int i = 0; i < NST; ++i) {
-      mbar_init(&sm.qd_full[i], 1);
-      mbar_init(&sm.qd_empty[i], 1);
-      mbar_init(&sm.dp_full[i], 1);
-      mbar_init(&sm.ds_free[i], 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.q_full[i], 1);
+      mbar_init(&sm.q_empty[i], 1);
     }
+    mbar_init(&sm.do_full, 1);
+    mbar_init(&sm.do_empty, 1);
     mbar_init(&sm.s_full, 1);
-    mbar_init(&sm.p_ready, 256);
-    mbar_init(&sm.s_read, 256);
+    mbar_init(&sm.dp_full, 1);
+    mbar_init(&sm.p_ready, 128);
     mbar_init(&sm.dq_full, 1);
-    mbar_init(&sm.dq_free, 128);
+    mbar_init(&sm.dq_free, 256);
     mbar_init(&sm.kv_done, 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
@@ -123,178 +131,182 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         tma_load_5d(sm.k + c * BK * 64, &P.tm_k, &sm.kv_full, c * 64, kvh, s, n0, b);
         tma_load_5d(sm.v + c * BK * 64, &P.tm_v, &sm.kv_full, c * 64, kvh, s, n0, b);
       }
-      int issued = 0;
-      for (int t = 0; t < T; ++t, ++issued) {
-        const int st = t & 1;
-        if (t >= NST && !mbar_wait(&sm.qd_empty[st], ((t - NST) >> 1) & 1, abort, P.status)) break;
+      int nq_issued = 0, ndo_issued = 0;
+      // query tiles run up to two ahead (double buffer); dO / lse2 / delta one ahead
+      for (int t = 0; t < T; ++t) {
         const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
-        mbar_arrive_expect_tx(&sm.qd_full[st], 2 * BQ * DH * 2 + 2 * BQ * 4);
-        for (int c = 0; c < DH / 64; ++c) {
-          tma_load_5d(sm.q[st] + c * BQ * 64, &P.tm_q, &sm.qd_full[st], c * 64, h, s, q0, b);
-          tma_load_5d(sm.dO[st] + c * BQ * 64, &P.tm_do, &sm.qd_full[st], c * 64, h, s, q0, b);
-        }
+        const int qb = t & 1;
+        if (t >= 2 && !mbar_wait(&sm.q_empty[qb], ((t - 2) >> 1) & 1, abort, P.status)) break;
+        mbar_arrive_expect_tx(&sm.q_full[qb], BQ * DH * 2);
+        for (int c = 0; c < DH / 64; ++c)
+          tma_load_5d(sm.q[qb] + c * BQ * 64, &P.tm_q, &sm.q_full[qb], c * 64, h, s, q0, b);
+        ++nq_issued;
+        if (t >= 1 && !mbar_wait(&sm.do_empty, (t - 1) & 1, abort, P.status)) break;
+        mbar_arrive_expect_tx(&sm.do_full, BQ * DH * 2 + 2 * BQ * 4);
+        for (int c = 0; c < DH / 64; ++c)
+          tma_load_5d(sm.dO + c * BQ * 64, &P.tm_do, &sm.do_full, c * 64, h, s, q0, b);
         const long long off = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + q0;
-        bulk_load(sm.lse2[st], P.lse2 + off, BQ * 4, &sm.qd_full[st]);
-        bulk_load(sm.delta[st], P.delta + off, BQ * 4, &sm.qd_full[st]);
+        bulk_load(sm.lse2, P.lse2 + off, BQ * 4, &sm.do_full);
+        bulk_load(sm.delta, P.delta + off, BQ * 4, &sm.do_full);
+        ++ndo_issued;
       }
+      // every copy this thread started lands before the CTA may exit
       mbar_drain(&sm.kv_full, 0);
-      for (int t = max(0, issued - NST); t < issued; ++t) mbar_drain(&sm.qd_full[t & 1], (t >> 1) & 1);
+      for (int t = max(0, nq_issued - 2); t < nq_issued; ++t) mbar_drain(&sm.q_full[t & 1], (t >> 1) & 1);
+      if (ndo_issued > 0) mbar_drain(&sm.do_full, (ndo_issued - 1) & 1);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idS = idesc_bf16(128, BQ, 0, 0);   // S^T, dP^T: A = K/V, B = Q/dO (K-major)
-      constexpr uint32_t idKV = idesc_bf16(128, DH, 0, 1);  // dV, dK: A in TMEM, B = dO/Q MN-major
-      constexpr uint32_t idQ = idesc_bf16(128, BQ, 1, 1);   // dQ^T: A = K^T, B = dS^T, both MN-major
-      const uint32_t ka = smem_u32(sm.k), va = smem_u32(sm.v);
-      // S^T = K Q^T or dP^T = V dO^T of tile t into TMEM column col
-      auto issue_sdp = [&](uint32_t aa, const bf16* bt, uint32_t col) {
-        const uint32_t ba = smem_u32(bt);
+      constexpr uint32_t idSP = idesc_bf16(128, BQ, 0, 0);  // S^T, dP^T: A = K / V, B = Q / dO (K-major)
+      constexpr uint32_t idKV = idesc_bf16(128, DH, 0, 1);  // dV, dK: A in TMEM, B = dO / Q MN-major
+      constexpr uint32_t idQ = idesc_bf16(128, DH, 1, 1);   // dQ: A = dS (dS^T tile MN-major), B = K MN-major
+      const uint32_t ka = smem_u32(sm.k), va = smem_u32(sm.v), da = smem_u32(sm.dO), dsa = smem_u32(sm.ds);
+      auto issue_sp = [&](uint32_t aa, uint32_t ba, uint32_t col) {
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
           const uint64_t ad = sdesc_sw128(aa + (kk >> 2) * (BK * 128) + (kk & 3) * 32, 16, 1024);
           const uint64_t bd = sdesc_sw128(ba + (kk >> 2) * (BQ * 128) + (kk & 3) * 32, 16, 1024);
-          tc_mma_ss(tmem + col, ad, bd, idS, kk > 0 ? 1u : 0u);
+          tc_mma_ss(tmem + col, ad, bd, idSP, kk > 0 ? 1u : 0u);
         }
       };
-      // dV (a_col = P^T) or dK (a_col = dS^T) += A * B, B = dO or Q of the tile (MN-major)
-      auto issue_kv = [&](uint32_t a_col, const bf16* bt, uint32_t d_col, bool acc) {
-        const uint32_t ba = smem_u32(bt);
+      // dV (a_col = P^T) or dK (a_col = dS^T) += A * B; B = dO or Q [query rows][d], MN-major
+      auto issue_kv = [&](uint32_t a_col, uint32_t ba, uint32_t d_col, bool acc) {
 #pragma unroll
         for (int kk = 0; kk < BQ / 16; ++kk) {
           const uint64_t bd = sdesc_sw128(ba + kk * 16 * 128, BQ * 128, 1024);
           tc_mma_ts(tmem + d_col, tmem + a_col + kk * 8, bd, idKV, (acc || kk > 0) ? 1u : 0u);
         }
       };
-      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.qd_full[0], 0, abort, P.status);
+      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.q_full[0], 0, abort, P.status);
       if (ok) {
         tc_fence_after();
-        issue_sdp(ka, sm.q[0], COL_ST);
+        issue_sp(ka, smem_u32(sm.q[0]), col_r(0));
         tc_commit(&sm.s_full);
-        issue_sdp(va, sm.dO[0], col_dpt(0));
-        tc_commit(&sm.dp_full[0]);
+        ok = mbar_wait(&sm.do_full, 0, abort, P.status);
+        if (ok) {
+          tc_fence_after();
+          issue_sp(va, da, col_r(1));
+          tc_commit(&sm.dp_full);
+        }
       }
       for (int t = 0; ok && t < T; ++t) {
-        const int st = t & 1, sn = st ^ 1;
-        if (t + 1 < T) {
-          // dP^T(t+1): its columns last held dS^T(t-1), read by dK(t-1) issued earlier
-          if (!mbar_wait(&sm.qd_full[sn], ((t + 1) >> 1) & 1, abort, P.status)) { ok = false; break; }
-          tc_fence_after();
-          issue_sdp(va, sm.dO[sn], col_dpt(sn));
-          tc_commit(&sm.dp_full[sn]);
-        }
+        const int p = t & 1;
+        const uint32_t qa = smem_u32(sm.q[p]);
         if (!mbar_wait(&sm.p_ready, t & 1, abort, P.status)) { ok = false; break; }
         tc_fence_after();
-        issue_kv(COL_ST, sm.dO[st], COL_DV, t > 0);
-        if (t + 1 < T) {
-          issue_sdp(ka, sm.q[sn], COL_ST);  // after dV(t) read P^T(t)
-          tc_commit(&sm.s_full);
-        }
-        issue_kv(col_dpt(st), sm.q[st], COL_DK, t > 0);
-        tc_commit(&sm.qd_empty[st]);
-        if (t >= 1 && !mbar_wait(&sm.dq_free, (t - 1) & 1, abort, P.status)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t dsa = smem_u32(sm.ds[st]);
+        issue_kv(col_r(p), da, COL_DV, t > 0);        // reads P^T(t) and dO(t)
+        tc_commit(&sm.do_empty);
+        issue_kv(col_r(p ^ 1), qa, COL_DK, t > 0);    // reads dS^T(t) and Q(t)
+        tc_commit(&sm.q_empty[p]);
+        // dQ(t) = dS K into R[p] (after dV(t) read P^T there)
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(ka + kk * 16 * 128, BK * 128, 1024);
-          const uint64_t bd = sdesc_sw128(dsa + kk * 16 * 128, BK * 128, 1024);
-          tc_mma_ss(tmem + COL_DQ, ad, bd, idQ, kk > 0 ? 1u : 0u);
+          const uint64_t ad = sdesc_sw128(dsa + kk * 16 * 128, BK * 128, 1024);
+          const uint64_t bd = sdesc_sw128(ka + kk * 16 * 128, BK * 128, 1024);
+          tc_mma_ss(tmem + col_r(p), ad, bd, idQ, kk > 0 ? 1u : 0u);
         }
         tc_commit(&sm.dq_full);
-        tc_commit(&sm.ds_free[st]);
+        if (t + 1 < T) {
+          // S^T(t+1) into R[p^1]: dK(t) has read dS^T(t) from it
+          if (!mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status)) { ok = false; break; }
+          tc_fence_after();
+          issue_sp(ka, smem_u32(sm.q[p ^ 1]), col_r(p ^ 1));
+          tc_commit(&sm.s_full);
+          // dP^T(t+1) into R[p]: dQ(t) must have been read out, dO(t+1) loaded
+          if (!mbar_wait(&sm.dq_free, t & 1, abort, P.status) ||
+              !mbar_wait(&sm.do_full, (t + 1) & 1, abort, P.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_sp(va, da, col_r(p));
+          tc_commit(&sm.dp_full);
+        }
       }
       tc_commit(&sm.kv_done);
       tc_commit(&sm.drain);
       mbar_drain(&sm.drain, 0);
     }
-  } else if (warp < 10) {
-    // ------------------------------------------------------------ softmax (key rows)
-    const int half = (warp - 2) >> 2;  // query columns [32*half, 32*half + 32)
+  } else if (warp < 6) {
+    // ------------------------------------------------------------ softmax
     const int q4 = warp & 3;
-    const int row = q4 * 32 + lane;
+    const int row = q4 * 32 + lane;    // TMEM lane
     const int kr = n0 + row;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     const float c2 = P.scale_log2;
+    uint8_t* dsrow = reinterpret_cast<uint8_t*>(sm.ds) + row * 128;
     bool ok = true;
     for (int t = 0; t < T; ++t) {
-      const int st = t & 1;
-      const int q0 = (i_lo + t % nq) * BQ + 32 * half;
+      const int p = t & 1;
+      const int q0 = (i_lo + t % nq) * BQ;
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status) &&
-                                       mbar_wait(&sm.dp_full[st], (t >> 1) & 1, abort, P.status))) {
+                                       mbar_wait(&sm.dp_full, t & 1, abort, P.status) &&
+                                       mbar_wait(&sm.do_full, t & 1, abort, P.status))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      uint32_t sr[32], dr[32];
-      tmem_ld32(tl + COL_ST + 32 * half, sr);
-      tmem_ld32(tl + col_dpt(st) + 32 * half, dr);
-      tmem_ld_wait();
-      // both halves have read their S^T / dP^T columns before either packs bf16 over them
-      // (an mbarrier rather than bar.sync, so an aborted peer cannot strand this warp)
-      tc_fence_before();
-      mbar_arrive(&sm.s_read);
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_read, t & 1, abort, P.status))) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const float4* l2 = reinterpret_cast<const float4*>(sm.lse2[st] + 32 * half);
-      const float4* dl = reinterpret_cast<const float4*>(sm.delta[st] + 32 * half);
-      const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + 32 > G.Lv);
-      if (need_mask) {
-        // zero the scores of invisible pairs up front: exp2(-inf) = 0 below
+      const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + BQ > G.Lv);
+      // four chunks of 32 query columns; chunk c packs into columns [16c, 16c+16),
+      // which hold data of chunks this thread has already read
 #pragma unroll
-        for (int c = 0; c < 32; ++c)
-          if (!visible(q0 + c, kr, G.Lv, G.window)) sr[c] = __float_as_uint(-INFINITY);
-      }
-      uint32_t pp[16], dd[16];
+      for (int c = 0; c < 4; ++c) {
+        const uint32_t cs = col_r(p) + 32 * c, cd = col_r(p ^ 1) + 32 * c;
+        uint32_t sr[32], dr[32];
+        tmem_ld32(tl + cs, sr);
+        tmem_ld32(tl + cd, dr);
+        tmem_ld_wait();
+        const int qb = q0 + 32 * c;
+        if (need_mask) {
 #pragma unroll
-      for (int c4 = 0; c4 < 8; ++c4) {
-        const float4 lv = l2[c4], dv = dl[c4];
-        const float la[4] = {lv.x, lv.y, lv.z, lv.w}, da[4] = {dv.x, dv.y, dv.z, dv.w};
-        float p[4], d[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int c = c4 * 4 + e;
-          p[e] = ex2_approx(fmaf(__uint_as_float(sr[c]), c2, -la[e]));
-          d[e] = p[e] * (__uint_as_float(dr[c]) - da[e]);
+          for (int e = 0; e < 32; ++e)
+            if (!visible(qb + e, kr, G.Lv, G.window)) sr[e] = __float_as_uint(-INFINITY);
         }
-        pp[2 * c4] = cvt_bf16x2(p[0], p[1]);
-        pp[2 * c4 + 1] = cvt_bf16x2(p[2], p[3]);
-        dd[2 * c4] = cvt_bf16x2(d[0], d[1]);
-        dd[2 * c4 + 1] = cvt_bf16x2(d[2], d[3]);
-      }
-      // P^T and dS^T (bf16 pairs) over the first 32 columns of S^T and dP^T[st]
-      tmem_st16(tl + COL_ST + 16 * half, pp);
-      tmem_st16(tl + col_dpt(st) + 16 * half, dd);
-      // dS^T -> shared memory for the dQ MMA; this buffer was last read by dQ(t-2)
-      if (t >= NST &&
-          !__all_sync(0xffffffffu, mbar_wait(&sm.ds_free[st], ((t - NST) >> 1) & 1, abort, P.status))) {
-        ok = false;
-        break;
-      }
-      uint8_t* dsrow = reinterpret_cast<uint8_t*>(sm.ds[st]) + row * 128;
+        const float4* l2 = reinterpret_cast<const float4*>(sm.lse2 + 32 * c);
+        const float4* dl = reinterpret_cast<const float4*>(sm.delta + 32 * c);
+        uint32_t pp[16], dd[16];
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
-        *reinterpret_cast<uint4*>(dsrow + (((4 * half + c) ^ (row & 7)) << 4)) =
-            make_uint4(dd[4 * c], dd[4 * c + 1], dd[4 * c + 2], dd[4 * c + 3]);
+        for (int c4 = 0; c4 < 8; ++c4) {
+          const float4 lv = l2[c4], dv = dl[c4];
+          const float la[4] = {lv.x, lv.y, lv.z, lv.w}, dla[4] = {dv.x, dv.y, dv.z, dv.w};
+          float pv[4], dsv[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            pv[e] = ex2_approx(fmaf(__uint_as_float(sr[c4 * 4 + e]), c2, -la[e]));
+            dsv[e] = pv[e] * (__uint_as_float(dr[c4 * 4 + e]) - dla[e]);
+          }
+          pp[2 * c4] = cvt_bf16x2(pv[0], pv[1]);
+          pp[2 * c4 + 1] = cvt_bf16x2(pv[2], pv[3]);
+          dd[2 * c4] = cvt_bf16x2(dsv[0], dsv[1]);
+          dd[2 * c4 + 1] = cvt_bf16x2(dsv[2], dsv[3]);
+        }
+        // packed P^T / dS^T for query columns [32c, +32): TMEM columns [16c, +16)
+        tmem_st16(tl + col_r(p) + 16 * c, pp);
+        tmem_st16(tl + col_r(p ^ 1) + 16 * c, dd);
+        // dS^T -> shared memory for dQ(t): block c/2, 16-byte chunks 4(c%2)..4(c%2)+3
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          *reinterpret_cast<uint4*>(dsrow + (c >> 1) * (BK * 128) + (((4 * (c & 1) + k) ^ (row & 7)) << 4)) =
+              make_uint4(dd[4 * k], dd[4 * k + 1], dd[4 * k + 2], dd[4 * k + 3]);
+      }
       fence_async_smem();
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(&sm.p_ready);
     }
-    // epilogue: half 0 writes this key row of dV, half 1 of dK (scaled)
+    // epilogue: this key row of dV, then of dK (scaled)
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
       tc_fence_after();
       const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + s) * G.Hkv + kvh) * DH;
-      const float mul = half ? P.scale : 1.f;
-      bf16* dst = (half ? P.dk : P.dv) + orow;
-      const uint32_t col = half ? COL_DK : COL_DV;
-#pragma unroll
-      for (int c = 0; c < DH / 32; ++c) {
+#pragma unroll 1
+      for (int c = 0; c < 2 * DH / 32; ++c) {
+        const int which = c >= DH / 32;
+        const float mul = which ? P.scale : 1.f;
+        bf16* dst = (which ? P.dk : P.dv) + orow + (c % (DH / 32)) * 32;
+        const uint32_t col = (which ? COL_DK : COL_DV) + (c % (DH / 32)) * 32;
         uint32_t o[32];
-        tmem_ld32(tl + col + c * 32, o);
+        tmem_ld32(tl + col, o);
         tmem_ld_wait();
         if (kr < G.Lv) {
 #pragma unroll
@@ -304,36 +316,51 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
             w.y = cvt_bf16x2(__uint_as_float(o[e + 2]) * mul, __uint_as_float(o[e + 3]) * mul);
             w.z = cvt_bf16x2(__uint_as_float(o[e + 4]) * mul, __uint_as_float(o[e + 5]) * mul);
             w.w = cvt_bf16x2(__uint_as_float(o[e + 6]) * mul, __uint_as_float(o[e + 7]) * mul);
-            *reinterpret_cast<uint4*>(dst + c * 32 + e) = w;
+            *reinterpret_cast<uint4*>(dst + e) = w;
           }
         }
       }
     }
   } else {
-    // ------------------------------------------------------------ dQ flush (head-dim rows)
+    // ------------------------------------------------------------ dQ flush
+    // TMEM lane = query row q0 + 32*q4 + lane; this warp's 64 head-dim columns leave
+    // TMEM first, then two 32-column rounds are staged (128-byte swizzle) and added
+    // into the fp32 accumulator by TMA reduce.
+    const int dhalf = (warp - 6) >> 2;
     const int q4 = warp & 3;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
-    float* stage = sm.dq[q4];
-    for (int t = 0; t < T; ++t) {
+    float* stage = sm.dqs[warp - 6];
+    bool ok = true;
+    for (int t = 0; ok && t < T; ++t) {
+      const int p = t & 1;
       const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) {
+        ok = false;
+        break;
+      }
       tc_fence_after();
-      uint32_t v[BQ];
-      tmem_ld32(tl + COL_DQ, v);
-      tmem_ld32(tl + COL_DQ + 32, v + 32);
+      uint32_t v[64];
+      tmem_ld32(tl + col_r(p) + 64 * dhalf, v);
+      tmem_ld32(tl + col_r(p) + 64 * dhalf + 32, v + 32);
       tmem_ld_wait();
       tc_fence_before();
-      mbar_arrive(&sm.dq_free);
-      // the previous reduce must have finished reading the staging buffer
-      if (lane == 0) bulk_wait_read0();
-      __syncwarp();
+      mbar_arrive(&sm.dq_free);  // the MMA may now overwrite these columns
 #pragma unroll
-      for (int c = 0; c < BQ; ++c) stage[c * 32 + lane] = __uint_as_float(v[c]);
-      fence_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        tma_reduce_add_5d(&P.tm_dq, stage, q4 * 32, h, s, q0, b);
-        bulk_commit();
+      for (int r2 = 0; r2 < 2; ++r2) {
+        // the previous reduce from this warp's buffer must have read it
+        if (lane == 0) bulk_wait_read0();
+        __syncwarp();
+        uint8_t* srow = reinterpret_cast<uint8_t*>(stage) + lane * 128;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          *reinterpret_cast<uint4*>(srow + ((c ^ (lane & 7)) << 4)) =
+              make_uint4(v[32 * r2 + 4 * c], v[32 * r2 + 4 * c + 1], v[32 * r2 + 4 * c + 2], v[32 * r2 + 4 * c + 3]);
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_reduce_add_5d(&P.tm_dq, stage, 64 * dhalf + 32 * r2, h, s, q0 + q4 * 32, b);
+          bulk_commit();
+        }
       }
     }
     if (lane == 0) bulk_wait0();
@@ -357,7 +384,7 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   Params p;
   if (!make_rows_tmap(&p.tm_q, q, g, g.Hq, DH, BQ) || !make_rows_tmap(&p.tm_do, dout, g, g.Hq, DH, BQ) ||
       !make_rows_tmap(&p.tm_k, k, g, g.Hkv, DH, BK) || !make_rows_tmap(&p.tm_v, v, g, g.Hkv, DH, BK) ||
-      !make_rows_tmap(&p.tm_dq, dq_ws, g, g.Hq, DH, BQ, 4, 32, false))
+      !make_rows_tmap(&p.tm_dq, dq_ws, g, g.Hq, DH, 32, 4, 32, true))
     return cudaErrorInvalidValue;
   p.lse2 = lse2_ws;
   p.delta = delta_ws;

@@ -102,6 +102,7 @@ HD_DEVINLINE void tma_reduce_add_5d(const CUtensorMap* m, const void* src, int c
 }
 HD_DEVINLINE void bulk_commit() { asm volatile("cp.async.bulk.commit_group;\n" ::: "memory"); }
 HD_DEVINLINE void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory"); }
+HD_DEVINLINE void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;\n" ::: "memory"); }
 HD_DEVINLINE void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory"); }
 
 // ---------------------------------------------------------------- tcgen05
