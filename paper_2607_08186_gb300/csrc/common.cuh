@@ -22,6 +22,11 @@ struct SfaGeom {
   int window;   // > 0 only for LOCAL: key r' visible iff r - window < r' <= r
 };
 
+// Stream-major backward row terms (-lse*log2e, -delta) are padded per (b, h, stream)
+// to a multiple of the largest query tile any backward kernel reads at once.
+constexpr int kRowTermAlign = 128;
+__host__ __device__ inline int row_terms_pitch(int Lv) { return (Lv + kRowTermAlign - 1) / kRowTermAlign * kRowTermAlign; }
+
 HD_DEVINLINE uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -76,8 +76,8 @@ float resolve_scale(float s, int Dh) { return s > 0.f ? s : 1.0f / sqrtf((float)
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then lse*log2(e) and
-// delta, each fp32 [B][Hq][ns][Lvp] (stream-major rows, Lvp = Lv rounded up to 64).
+// Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then -lse*log2(e) and
+// -delta, each fp32 [B][Hq][ns][Lvp] (stream-major rows, Lvp = row_terms_pitch(Lv)).
 struct BwdWs {
   float* dq;
   float* lse2;
@@ -86,7 +86,7 @@ struct BwdWs {
 
 size_t ws_bytes(const SfaGeom& g, int Dh) {
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
-  const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)((g.Lv + 63) & ~63);
+  const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)row_terms_pitch(g.Lv);
   return align256(rows * Dh * sizeof(float)) + 2 * align256(trows * sizeof(float));
 }
 
@@ -94,7 +94,7 @@ hd_status_t split_ws(const SfaGeom& g, int Dh, void* ws, size_t bytes, BwdWs* ou
   if (ws == nullptr || bytes < ws_bytes(g, Dh) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
     return HD_ERR_WORKSPACE;
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
-  const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)((g.Lv + 63) & ~63);
+  const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)row_terms_pitch(g.Lv);
   char* p = static_cast<char*>(ws);
   out->dq = reinterpret_cast<float*>(p);
   p += align256(rows * Dh * sizeof(float));

@@ -1,10 +1,11 @@
 // Backward pre- and post-processing (bandwidth kernels).
 //
-// prep:     delta[p] = sum_d dO[p,d] * O[p,d] (fp32) and lse2[p] = lse[p] * log2(e),
+// prep:     -delta[p] = -sum_d dO[p,d] * O[p,d] (fp32) and -lse2[p] = -lse[p] * log2(e),
 //           both written stream-major, [B][Hq][ns][Lvp] with row r of stream s at
-//           position p = r*ns + s and Lvp = Lv rounded up to 64, so one query tile
-//           of any stream is 64 contiguous floats (a single bulk copy).  Rows in
-//           [Lv, Lvp) get lse2 = +inf and delta = 0 (their P and dS vanish).
+//           position p = r*ns + s and Lvp = row_terms_pitch(Lv), so one query tile
+//           of any stream is contiguous floats (a single bulk copy).  Negated so the
+//           backward folds them in with one add / fused multiply-add.  Rows in
+//           [Lv, Lvp) get -lse2 = -inf and -delta = 0 (their P and dS vanish).
 //           Also zeroes the fp32 dQ accumulator.
 // finalize: dq = bf16(scale * accumulator), round to nearest even.
 #include "common.cuh"
@@ -38,20 +39,20 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
   for (int c = lane; c < DH / 4; c += 32) dqr[c] = make_float4(0.f, 0.f, 0.f, 0.f);
   if (lane == 0) {
     const long long h = row % g.Hq, bp = row / g.Hq, p = bp % g.nL, b = bp / g.nL;
-    const int Lvp = (g.Lv + 63) & ~63;
+    const int Lvp = row_terms_pitch(g.Lv);
     const long long s = p % g.ns, r = p / g.ns;
     const long long t = ((b * g.Hq + h) * g.ns + s) * Lvp + r;
-    delta_t[t] = acc;
-    lse2_t[t] = lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
+    delta_t[t] = -acc;
+    lse2_t[t] = -lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
   }
 }
 
 __global__ void sfa_bwd_pad_kernel(float* __restrict__ lse2_t, float* __restrict__ delta_t, SfaGeom g) {
-  const int Lvp = (g.Lv + 63) & ~63, pad = Lvp - g.Lv;
+  const int Lvp = row_terms_pitch(g.Lv), pad = Lvp - g.Lv;
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (long long)g.B * g.Hq * g.ns * pad) return;
   const long long t = (i / pad) * Lvp + g.Lv + i % pad;
-  lse2_t[t] = INFINITY;
+  lse2_t[t] = -INFINITY;
   delta_t[t] = 0.f;
 }
 
@@ -83,7 +84,7 @@ cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* ls
                                                     delta_ws, dq_ws, g);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int pad = ((g.Lv + 63) & ~63) - g.Lv;
+  const int pad = row_terms_pitch(g.Lv) - g.Lv;
   if (pad > 0) {
     const long long n = (long long)g.B * g.Hq * g.ns * pad;
     sfa_bwd_pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(lse2_ws, delta_ws, g);

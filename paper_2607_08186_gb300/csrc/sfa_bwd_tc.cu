@@ -7,7 +7,8 @@
 // also within the window).  Every GEMM is a 128 x 128 x 16k tcgen05 MMA (N = 128
 // runs at full tensor rate; N = 64 does not):
 //   S^T  = K Q^T,  dP^T = V dO^T        SS: A = K / V (K-major), B = Q / dO (K-major)
-//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)      (softmax)
+//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)      (softmax;
+//                                       packed f32x2 arithmetic, exp2 on the SFU)
 //   dV  += P^T dO,  dK += dS^T Q        TS: A = P^T / dS^T packed bf16 in TMEM
 //   dQ   = dS K                         SS: A = dS^T tile in smem read MN-major,
 //                                           B = K read MN-major; TMEM lane = query row
@@ -26,7 +27,7 @@
 //
 // Roles (448 threads, at most 4 warps per scheduler so each thread keeps 128
 // registers): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer, warps 2..5
-// softmax (TMEM lane = key row; 128 query columns in four 32-column chunks),
+// softmax (TMEM lane = key row; 128 query columns in eight 16-column chunks),
 // warps 6..9 / 10..13 dQ flush for head-dim columns 0..63 / 64..127 (TMEM lane =
 // query row): each loads its 64 columns, releases the TMEM, then stages two 4 KB
 // rounds through its own buffer.
@@ -89,7 +90,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
   if (G.window > 0) i_hi = min(i_hi, (n0 + BK - 1 + G.window - 1) / BQ);
   const int nq = i_hi - i_lo + 1;
   const int T = grp * nq;
-  const int Lvp = (G.Lv + 63) & ~63;
+  const int Lvp = row_terms_pitch(G.Lv);
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.kv_full, 1);
@@ -248,46 +249,57 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       }
       tc_fence_after();
       const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + BQ > G.Lv);
-      // four chunks of 32 query columns; chunk c packs into columns [16c, 16c+16),
-      // which hold data of chunks this thread has already read
+      // eight chunks of 16 query columns; the TMEM loads of chunk c+1 are in flight
+      // while chunk c is computed.  Chunk c packs into columns [8c, 8c+8), which hold
+      // data of chunks this thread has already read (and no chunk still to be loaded).
+      const uint64_t c2x2 = f2pack(c2, c2);
+      uint32_t sbuf[2][16], dbuf[2][16];
+      tmem_ld16(tl + col_r(p), sbuf[0]);
+      tmem_ld16(tl + col_r(p ^ 1), dbuf[0]);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const uint32_t cs = col_r(p) + 32 * c, cd = col_r(p ^ 1) + 32 * c;
-        uint32_t sr[32], dr[32];
-        tmem_ld32(tl + cs, sr);
-        tmem_ld32(tl + cd, dr);
-        tmem_ld_wait();
-        const int qb = q0 + 32 * c;
+      for (int c = 0; c < 8; ++c) {
+        uint32_t* sr = sbuf[c & 1];
+        uint32_t* dr = dbuf[c & 1];
+        tmem_ld_wait();  // chunk c has landed (the only loads in flight)
+        if (c + 1 < 8) {
+          tmem_ld16(tl + col_r(p) + 16 * (c + 1), sbuf[(c + 1) & 1]);
+          tmem_ld16(tl + col_r(p ^ 1) + 16 * (c + 1), dbuf[(c + 1) & 1]);
+        }
         if (need_mask) {
 #pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (!visible(qb + e, kr, G.Lv, G.window)) sr[e] = __float_as_uint(-INFINITY);
+          for (int e = 0; e < 16; ++e)
+            if (!visible(q0 + 16 * c + e, kr, G.Lv, G.window)) sr[e] = __float_as_uint(-INFINITY);
         }
-        const float4* l2 = reinterpret_cast<const float4*>(sm.lse2 + 32 * c);
-        const float4* dl = reinterpret_cast<const float4*>(sm.delta + 32 * c);
-        uint32_t pp[16], dd[16];
+        // sm.lse2 / sm.delta hold -lse*log2(e) and -delta (see sfa_bwd_prep.cu)
+        const float4* l2 = reinterpret_cast<const float4*>(sm.lse2 + 16 * c);
+        const float4* dl = reinterpret_cast<const float4*>(sm.delta + 16 * c);
+        uint32_t pp[8], dd[8];
 #pragma unroll
-        for (int c4 = 0; c4 < 8; ++c4) {
+        for (int c4 = 0; c4 < 4; ++c4) {
           const float4 lv = l2[c4], dv = dl[c4];
-          const float la[4] = {lv.x, lv.y, lv.z, lv.w}, dla[4] = {dv.x, dv.y, dv.z, dv.w};
-          float pv[4], dsv[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            pv[e] = ex2_approx(fmaf(__uint_as_float(sr[c4 * 4 + e]), c2, -la[e]));
-            dsv[e] = pv[e] * (__uint_as_float(dr[c4 * 4 + e]) - dla[e]);
+          for (int hp = 0; hp < 2; ++hp) {
+            const int e = 4 * c4 + 2 * hp;
+            float x0, x1;
+            f2unpack(ffma2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2,
+                           hp ? f2pack(lv.z, lv.w) : f2pack(lv.x, lv.y)),
+                     x0, x1);
+            const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+            const uint64_t dpd = fadd2(f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1])),
+                                       hp ? f2pack(dv.z, dv.w) : f2pack(dv.x, dv.y));
+            float d0, d1;
+            f2unpack(fmul2(f2pack(p0, p1), dpd), d0, d1);
+            pp[e >> 1] = cvt_bf16x2(p0, p1);
+            dd[e >> 1] = cvt_bf16x2(d0, d1);
           }
-          pp[2 * c4] = cvt_bf16x2(pv[0], pv[1]);
-          pp[2 * c4 + 1] = cvt_bf16x2(pv[2], pv[3]);
-          dd[2 * c4] = cvt_bf16x2(dsv[0], dsv[1]);
-          dd[2 * c4 + 1] = cvt_bf16x2(dsv[2], dsv[3]);
         }
-        // packed P^T / dS^T for query columns [32c, +32): TMEM columns [16c, +16)
-        tmem_st16(tl + col_r(p) + 16 * c, pp);
-        tmem_st16(tl + col_r(p ^ 1) + 16 * c, dd);
-        // dS^T -> shared memory for dQ(t): block c/2, 16-byte chunks 4(c%2)..4(c%2)+3
+        tmem_st8(tl + col_r(p) + 8 * c, pp);
+        tmem_st8(tl + col_r(p ^ 1) + 8 * c, dd);
+        // dS^T -> shared memory for dQ(t): block c/4, 16-byte chunks 2(c%4), 2(c%4)+1
+        uint8_t* blk = dsrow + (c >> 2) * (BK * 128);
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          *reinterpret_cast<uint4*>(dsrow + (c >> 1) * (BK * 128) + (((4 * (c & 1) + k) ^ (row & 7)) << 4)) =
+        for (int k = 0; k < 2; ++k)
+          *reinterpret_cast<uint4*>(blk + (((2 * (c & 3) + k) ^ (row & 7)) << 4)) =
               make_uint4(dd[4 * k], dd[4 * k + 1], dd[4 * k + 2], dd[4 * k + 3]);
       }
       fence_async_smem();

@@ -32,8 +32,8 @@ struct MmaBwdArgs {
   const bf16* k;
   const bf16* v;
   const bf16* dout;
-  const float* lse2;   // [B][Hq][ns][Lvp] lse * log2(e), stream-major (see sfa_bwd_prep.cu)
-  const float* delta;  // [B][Hq][ns][Lvp] rowsum(dO * O)
+  const float* lse2;   // [B][Hq][ns][Lvp] -lse * log2(e), stream-major (see sfa_bwd_prep.cu)
+  const float* delta;  // [B][Hq][ns][Lvp] -rowsum(dO * O)
   float* dq_acc;       // [B][nL][Hq][Dh] fp32, pre-zeroed; gets sum dS K (unscaled)
   bf16* dk;
   bf16* dv;
@@ -233,8 +233,8 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   bf16* sQ = sV + BN * DH;                        // [2][BM][DH]
   bf16* sdO = sQ + 2 * BM * DH;                   // [2][BM][DH]
   bf16* sdS = sdO + 2 * BM * DH;                  // [BN][BM]  (dS^T, key-major)
-  float* sL = reinterpret_cast<float*>(sdS + BN * BM);  // [2][BM] lse * log2(e)
-  float* sD = sL + 2 * BM;                               // [2][BM] delta
+  float* sL = reinterpret_cast<float*>(sdS + BN * BM);  // [2][BM] -lse * log2(e)
+  float* sD = sL + 2 * BM;                               // [2][BM] -delta
 
   const SfaGeom G = a.g;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   auto q_base = [&](const bf16* t, int h) {
     return t + (((long long)b * G.nL + s) * G.Hq + h) * DH;
   };
-  const int Lvp = (G.Lv + 63) & ~63;
+  const int Lvp = row_terms_pitch(G.Lv);
   auto row_terms = [&](int it, int r, float& l2, float& dl) {
     const int h = kvh * grp + it / nq, m0 = (j + it % nq) * BM;
     const long long idx = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + m0 + r;
@@ -342,9 +342,9 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
           const int qr = m0 + ql;
           float p = 0.f;
           if (visible(qr, kr, G.Lv, G.window) && qr < G.Lv)
-            p = exp2f(sacc[i][e] * a.scale_log2 - cL[ql]);
+            p = exp2f(fmaf(sacc[i][e], a.scale_log2, cL[ql]));
           sacc[i][e] = p;
-          dpacc[i][e] = p * (dpacc[i][e] - cD[ql]);
+          dpacc[i][e] = p * (dpacc[i][e] + cD[ql]);
         }
       }
 #pragma unroll
