@@ -40,7 +40,8 @@ typedef enum {
   HD_ERR_CUDA = 3,        /* a CUDA runtime/driver call or kernel launch failed */
   HD_ERR_WORKSPACE = 4,   /* workspace null or smaller than sfa_bwd_workspace_bytes() */
   HD_ERR_TIMEOUT = 5,     /* reserved: a bounded device wait expired (see HD_DEVBIT_TIMEOUT) */
-  HD_ERR_INDEX = 6        /* reserved: an index was out of range (see HD_DEVBIT_INDEX) */
+  HD_ERR_INDEX = 6,       /* reserved: an index was out of range (see HD_DEVBIT_INDEX) */
+  HD_ERR_SCRATCH_LIMIT = 7 /* sfa_bwd_noalloc: sizes need more than SFA_BWD_NOALLOC_MAX_BYTES */
 } hd_status_t;
 
 /* Bits the kernels OR into *dev_status. */
@@ -120,6 +121,31 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
 hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
                              float softmax_scale, sfa_mode_t mode, void* workspace,
                              size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * sfa_bwd_noalloc -- sfa_bwd without a caller-supplied workspace.  The paper has no
+ * counterpart: this is an interface for callers that cannot hand the library device
+ * memory of their own (a runtime that commits its whole device-memory budget at
+ * start-up and forbids allocation while serving, or C code with no device allocator).
+ * Same arguments, outputs and status codes as sfa_bwd, minus the workspace.
+ *
+ * The workspace lives in a fixed device array of the library, SFA_BWD_NOALLOC_MAX_BYTES
+ * long, present in every CUDA context that loads the library's module; the call
+ * allocates and frees nothing.  Sizes whose sfa_bwd_workspace_bytes() exceeds that
+ * limit return HD_ERR_SCRATCH_LIMIT before anything is enqueued (use sfa_bwd there).
+ *   - Set-up: the first call on each device (current device at the time of the call)
+ *     looks up the array's device address and keeps it; make that first call before
+ *     any stream capture.  A failed look-up returns HD_ERR_CUDA.
+ *   - Sharing: every call on a device uses the same array, which keeps the last call's
+ *     contents; each call clears what it reads before reading it.  Calls that may run
+ *     concurrently on one device (unordered streams, several host threads) race on
+ *     the array: the caller must order them.
+ */
+#define SFA_BWD_NOALLOC_MAX_BYTES ((size_t)64 << 20)
+hd_status_t sfa_bwd_noalloc(const void* q, const void* k, const void* v, const void* o,
+                            const float* lse, const void* dout, void* dq, void* dk, void* dv, int B,
+                            int L, int n, int Hq, int Hkv, int Dh, float softmax_scale,
+                            sfa_mode_t mode, int window, int32_t* dev_status, cudaStream_t stream);
 
 /* Human-readable name of a status code (static string). */
 const char* hd_status_string(hd_status_t status);

@@ -55,6 +55,8 @@ def lib():
             L.sfa_bwd_main.argtypes = [P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
             L.sfa_bwd_finalize.restype = I
             L.sfa_bwd_finalize.argtypes = [P, I, I, I, I, I, I, F, I, P, Z, P]
+            L.sfa_bwd_noalloc.restype = I
+            L.sfa_bwd_noalloc.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, P]
             L.hd_status_string.restype = ctypes.c_char_p
             L.hd_status_string.argtypes = [I]
             _lib = L
@@ -119,6 +121,21 @@ def sfa_bwd(q, k, v, o, lse, dout, dq, dk, dv, n, mode, workspace, softmax_scale
                          B, L, n, Hq, Hkv, Dh, float(softmax_scale), int(mode), int(window),
                          _p(workspace), _wsb(workspace),
                          _p(dev_status), _stream(stream)), "sfa_bwd")
+    return dq, dk, dv
+
+
+SFA_BWD_NOALLOC_MAX_BYTES = 64 << 20
+
+
+def sfa_bwd_noalloc(q, k, v, o, lse, dout, dq, dk, dv, n, mode, softmax_scale=0.0, window=0,
+                    dev_status=None, stream=None):
+    """SFA backward with the library's fixed device workspace (no allocation anywhere,
+    at most SFA_BWD_NOALLOC_MAX_BYTES of workspace).  Calls on one device share that
+    workspace: order them (one stream, or events) so that none overlap."""
+    B, L, Hq, Hkv, Dh = _attn_dims(q, k, n)
+    _check(lib().sfa_bwd_noalloc(_p(q), _p(k), _p(v), _p(o), _p(lse), _p(dout), _p(dq), _p(dk),
+                                 _p(dv), B, L, n, Hq, Hkv, Dh, float(softmax_scale), int(mode),
+                                 int(window), _p(dev_status), _stream(stream)), "sfa_bwd_noalloc")
     return dq, dk, dv
 
 

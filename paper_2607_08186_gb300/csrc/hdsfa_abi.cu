@@ -216,6 +216,8 @@ const char* hd_status_string(hd_status_t s) {
     case HD_ERR_WORKSPACE: return "HD_ERR_WORKSPACE: workspace missing, misaligned or too small";
     case HD_ERR_TIMEOUT: return "HD_ERR_TIMEOUT: bounded device wait expired";
     case HD_ERR_INDEX: return "HD_ERR_INDEX: index out of range";
+    case HD_ERR_SCRATCH_LIMIT:
+      return "HD_ERR_SCRATCH_LIMIT: sizes need more workspace than sfa_bwd_noalloc's fixed array";
   }
   return "unknown hd_status_t";
 }
