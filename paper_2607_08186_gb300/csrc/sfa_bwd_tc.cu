@@ -20,7 +20,10 @@
 // TMEM: two 128-column regions R0, R1 swap roles with the tile parity p:
 //   S^T(t) in R[p] (P^T packed bf16 over its first 64 columns, then dQ(t)),
 //   dP^T(t) in R[p^1] (dS^T packed bf16 over its first 64 columns);  dV at 256, dK at 384.
-// MMA issue order:  wait P(t) | dV(t) dK(t) dQ(t) | S(t+1) | wait dQ(t) read-out | dP(t+1)
+// MMA issue order:  for each quarter u of the query columns: wait P(t) quarter u |
+//                   dV(t), dK(t) k-steps of quarter u;  then dQ(t) | S(t+1) |
+//                   wait dQ(t) read-out | dP(t+1)
+// so three quarters of dV(t), dK(t) run under the softmax of the later columns.
 // S(t+1) lands in R[p^1], whose dS^T(t) dK(t) has already consumed (tcgen05 MMAs of
 // one thread execute in order), so it overlaps the dQ(t) read-out; dP(t+1) lands in
 // R[p] only after that read-out.
@@ -52,7 +55,7 @@ struct Smem {
   float dqs[8][32 * 32];  // per dQ warp: [32 query rows][32 head-dim] fp32, 128-byte swizzle
   float lse2[BQ];
   float delta[BQ];
-  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, p_ready, dq_full, dq_free,
+  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, p_part[4], dq_full, dq_free,
       kv_done, drain;
   uint32_t tmem_base;
   int abort;
@@ -102,7 +105,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     mbar_init(&sm.do_empty, 1);
     mbar_init(&sm.s_full, 1);
     mbar_init(&sm.dp_full, 1);
-    mbar_init(&sm.p_ready, 128);
+    for (int i = 0; i < 4; ++i) mbar_init(&sm.p_part[i], 128);
     mbar_init(&sm.dq_full, 1);
     mbar_init(&sm.dq_free, 256);
     mbar_init(&sm.kv_done, 1);
@@ -171,10 +174,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
           tc_mma_ss(tmem + col, ad, bd, idSP, kk > 0 ? 1u : 0u);
         }
       };
-      // dV (a_col = P^T) or dK (a_col = dS^T) += A * B; B = dO or Q [query rows][d], MN-major
-      auto issue_kv = [&](uint32_t a_col, uint32_t ba, uint32_t d_col, bool acc) {
+      // dV (a_col = P^T) or dK (a_col = dS^T) += A * B over query k-steps [k0, k0+2);
+      // B = dO or Q [query rows][d], MN-major
+      auto issue_kv = [&](uint32_t a_col, uint32_t ba, uint32_t d_col, bool acc, int k0) {
 #pragma unroll
-        for (int kk = 0; kk < BQ / 16; ++kk) {
+        for (int kk = k0; kk < k0 + 2; ++kk) {
           const uint64_t bd = sdesc_sw128(ba + kk * 16 * 128, BQ * 128, 1024);
           tc_mma_ts(tmem + d_col, tmem + a_col + kk * 8, bd, idKV, (acc || kk > 0) ? 1u : 0u);
         }
@@ -194,11 +198,14 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       for (int t = 0; ok && t < T; ++t) {
         const int p = t & 1;
         const uint32_t qa = smem_u32(sm.q[p]);
-        if (!mbar_wait(&sm.p_ready, t & 1, abort, P.status)) { ok = false; break; }
-        tc_fence_after();
-        issue_kv(col_r(p), da, COL_DV, t > 0);        // reads P^T(t) and dO(t)
+        for (int u = 0; u < 4; ++u) {
+          if (!mbar_wait(&sm.p_part[u], t & 1, abort, P.status)) { ok = false; break; }
+          tc_fence_after();
+          issue_kv(col_r(p), da, COL_DV, t > 0, 2 * u);        // reads P^T(t) and dO(t)
+          issue_kv(col_r(p ^ 1), qa, COL_DK, t > 0, 2 * u);    // reads dS^T(t) and Q(t)
+        }
+        if (!ok) break;
         tc_commit(&sm.do_empty);
-        issue_kv(col_r(p ^ 1), qa, COL_DK, t > 0);    // reads dS^T(t) and Q(t)
         tc_commit(&sm.q_empty[p]);
         // dQ(t) = dS K into R[p] (after dV(t) read P^T there)
 #pragma unroll
@@ -301,11 +308,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         for (int k = 0; k < 2; ++k)
           *reinterpret_cast<uint4*>(blk + (((2 * (c & 3) + k) ^ (row & 7)) << 4)) =
               make_uint4(dd[4 * k], dd[4 * k + 1], dd[4 * k + 2], dd[4 * k + 3]);
+        if (c & 1) {
+          // query quarter c/2 packed: its dV / dK k-steps may start; after the last
+          // quarter the whole dS^T tile is also in shared memory for dQ(t)
+          if (c == 7) fence_async_smem();
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(&sm.p_part[c >> 1]);
+        }
       }
-      fence_async_smem();
-      tmem_st_wait();
-      tc_fence_before();
-      mbar_arrive(&sm.p_ready);
     }
     // epilogue: this key row of dV, then of dK (scaled)
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
