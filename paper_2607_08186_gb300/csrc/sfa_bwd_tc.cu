@@ -84,9 +84,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.x;  // key tile; tile 0 sees the most query tiles and starts first
+  // linear grid, key tile slowest: every CTA of key tile 0 (the most query tiles to
+  // visit) launches before any of tile 1, and so on, over all heads, streams and batches
+  const int per_tile = G.Hkv * G.ns * G.B;
+  const int j = (int)blockIdx.x / per_tile;
+  const int hsb = (int)blockIdx.x % per_tile;
   const int n0 = j * BK;
-  const int kvh = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
+  const int b = hsb / (G.Hkv * G.ns), kvh = (hsb / G.ns) % G.Hkv, s = hsb % G.ns;
   const int grp = G.Hq / G.Hkv;
   const int i_lo = n0 / BQ;
   int i_hi = (G.Lv - 1) / BQ;
@@ -420,7 +424,7 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   const int smem = (int)sizeof(Smem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((g.Lv + BK - 1) / BK, g.Hkv * g.ns, g.B);
+  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.ns * g.B);
   bwd_kernel<<<grid, NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }

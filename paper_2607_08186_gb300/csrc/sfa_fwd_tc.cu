@@ -70,9 +70,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ncta = (G.Lv + NG * BM - 1) / (NG * BM);
-  const int mt = ncta - 1 - (int)blockIdx.x;  // longest rows first
+  // linear grid, query-tile rank slowest: the last query tiles (the most key tiles to
+  // visit) of every head, stream and batch launch first
+  const int per_rank = G.Hq * G.ns * G.B;
+  const int mt = ncta - 1 - (int)blockIdx.x / per_rank;
+  const int hsb = (int)blockIdx.x % per_rank;
   const int m0 = mt * NG * BM;
-  const int h = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
+  const int b = hsb / (G.Hq * G.ns), h = (hsb / G.ns) % G.Hq, s = hsb % G.ns;
   const int kvh = h / (G.Hq / G.Hkv);
   int lo[NG], hi[NG];
 #pragma unroll
@@ -309,7 +313,8 @@ static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   const int smem = (int)sizeof(tcfwd::Smem<DH>) + 1024;
   cudaError_t e = cudaFuncSetAttribute(tcfwd::fwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((p.g.Lv + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM), p.g.Hq * p.g.ns, p.g.B);
+  const unsigned grid = (unsigned)((p.g.Lv + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM)) *
+                        (unsigned)(p.g.Hq * p.g.ns * p.g.B);
   tcfwd::fwd_kernel<DH><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }
