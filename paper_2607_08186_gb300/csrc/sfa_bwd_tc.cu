@@ -6,9 +6,12 @@
 // tiles that can see tile j (causal: query tiles at or after the key tile; LOCAL:
 // also within the window).  Every GEMM is a 128 x 128 x 16k tcgen05 MMA (N = 128
 // runs at full tensor rate; N = 64 does not):
-//   S^T  = K Q^T,  dP^T = V dO^T        SS: A = K / V (K-major), B = Q / dO (K-major)
-//   P^T  = exp2(S^T * scale*log2e - lse2),  dS^T = P^T (dP^T - delta)      (softmax;
-//                                       packed f32x2 arithmetic, exp2 on the SFU)
+//   S'^T = K Q^T - lse2/c2,  dP'^T = V dO^T - delta
+//                                       SS: A = K / V (K-major), B = Q / dO (K-major),
+//                                       accumulated onto TMEM pre-filled with the
+//                                       per-query terms (c2 = scale*log2e, lse2 = lse*log2e)
+//   P^T  = exp2(c2 S'^T),  dS^T = P^T dP'^T              (softmax; packed f32x2
+//                                       arithmetic, exp2 on the SFU, no shared memory)
 //   dV  += P^T dO,  dK += dS^T Q        TS: A = P^T / dS^T packed bf16 in TMEM
 //   dQ   = dS K                         SS: A = dS^T tile in smem read MN-major,
 //                                           B = K read MN-major; TMEM lane = query row
@@ -21,9 +24,12 @@
 //   S^T(t) in R[p] (P^T packed bf16 over its first 64 columns, then dQ(t)),
 //   dP^T(t) in R[p^1] (dS^T packed bf16 over its first 64 columns);  dV at 256, dK at 384.
 // MMA issue order:  for each quarter u of the query columns: wait P(t) quarter u |
-//                   dV(t), dK(t) k-steps of quarter u;  then dQ(t) | S(t+1) |
-//                   wait dQ(t) read-out | dP(t+1)
+//                   dV(t), dK(t) k-steps of quarter u;  then dQ(t) | wait R[p^1]
+//                   pre-filled | S(t+1) | wait dQ(t) read out and R[p] pre-filled | dP(t+1)
 // so three quarters of dV(t), dK(t) run under the softmax of the later columns.
+// The pre-fills (every TMEM lane gets the same 128 per-query values) are written
+// by the dQ warps: R[p^1] once dK(t) has read dS^T(t) (under dQ(t)), R[p] right
+// after they have read dQ(t) out of it.
 // S(t+1) lands in R[p^1], whose dS^T(t) dK(t) has already consumed (tcgen05 MMAs of
 // one thread execute in order), so it overlaps the dQ(t) read-out; dP(t+1) lands in
 // R[p] only after that read-out.
@@ -31,9 +37,9 @@
 // Roles (448 threads, at most 4 warps per scheduler so each thread keeps 128
 // registers): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer, warps 2..5
 // softmax (TMEM lane = key row; 128 query columns in eight 16-column chunks),
-// warps 6..9 / 10..13 dQ flush for head-dim columns 0..63 / 64..127 (TMEM lane =
-// query row): each loads its 64 columns, releases the TMEM, then stages two 4 KB
-// rounds through its own buffer.
+// warps 6..9 / 10..13 dQ flush and pre-fill for columns 0..63 / 64..127: each
+// loads its 64 dQ columns (TMEM lane = query row), pre-fills the region for the
+// next dP^T, then stages two 4 KB rounds through its own buffer.
 // Every mbarrier wait is bounded.
 #include "tc_common.cuh"
 
@@ -53,16 +59,18 @@ struct Smem {
   bf16 dO[BQ * DH];
   bf16 ds[BK * BQ];       // dS^T [128 key rows][128 queries]: 2 swizzle blocks of [128][64]
   float dqs[8][32 * 32];  // per dQ warp: [32 query rows][32 head-dim] fp32, 128-byte swizzle
-  float lse2[BQ];
-  float delta[BQ];
-  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, p_part[4], dq_full, dq_free,
-      kv_done, drain;
+  float nlse2[2][BQ];     // -lse*log2(e) of the query tile in q[i], loaded with it
+  float ndelta[2][BQ];    // -delta of the query tile in q[i], loaded with it
+  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, p_part[4], dq_full, s_init,
+      dp_init, dk_done, kv_done, drain;
   uint32_t tmem_base;
   int abort;
 };
 
-// dynamic shared memory (plus the 1 KB alignment pad) must fit the 227 KB per-block limit
-static_assert(sizeof(Smem) + 1024 <= 232448, "backward shared-memory layout exceeds 227 KB");
+// The layout, 1024-byte aligned inside the dynamic shared memory, must fit the 227 KB
+// per-block limit; the kernel checks the actual alignment pad on entry.
+constexpr int kSmemBytes = 232448;
+static_assert(sizeof(Smem) <= kSmemBytes, "backward shared-memory layout exceeds 227 KB");
 
 struct Params {
   CUtensorMap tm_q, tm_do, tm_k, tm_v, tm_dq;
@@ -81,6 +89,15 @@ HD_DEVINLINE bool visible(int r, int c, int Lv, int window) {
 
 __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant__ Params P) {
   extern __shared__ uint8_t smem_raw[];
+  {
+    uint32_t dyn;
+    asm("mov.u32 %0, %%dynamic_smem_size;\n" : "=r"(dyn));
+    const uintptr_t base = reinterpret_cast<uintptr_t>(smem_raw);
+    if (((base + 1023) & ~uintptr_t(1023)) - base + sizeof(Smem) > dyn) {  // uniform: nothing touched yet
+      if (threadIdx.x == 0) set_status(P.status, HD_DEVBIT_TIMEOUT);
+      return;
+    }
+  }
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -111,7 +128,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     mbar_init(&sm.dp_full, 1);
     for (int i = 0; i < 4; ++i) mbar_init(&sm.p_part[i], 128);
     mbar_init(&sm.dq_full, 1);
-    mbar_init(&sm.dq_free, 256);
+    mbar_init(&sm.s_init, 256);
+    mbar_init(&sm.dp_init, 256);
+    mbar_init(&sm.dk_done, 1);
     mbar_init(&sm.kv_done, 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
@@ -140,22 +159,22 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         tma_load_5d(sm.v + c * BK * 64, &P.tm_v, &sm.kv_full, c * 64, kvh, s, n0, b);
       }
       int nq_issued = 0, ndo_issued = 0;
-      // query tiles run up to two ahead (double buffer); dO / lse2 / delta one ahead
+      // query tiles (with their row terms) run up to two ahead (double buffer); dO one ahead
       for (int t = 0; t < T; ++t) {
         const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
         const int qb = t & 1;
         if (t >= 2 && !mbar_wait(&sm.q_empty[qb], ((t - 2) >> 1) & 1, abort, P.status)) break;
-        mbar_arrive_expect_tx(&sm.q_full[qb], BQ * DH * 2);
+        mbar_arrive_expect_tx(&sm.q_full[qb], BQ * DH * 2 + 2 * BQ * 4);
         for (int c = 0; c < DH / 64; ++c)
           tma_load_5d(sm.q[qb] + c * BQ * 64, &P.tm_q, &sm.q_full[qb], c * 64, h, s, q0, b);
+        const long long off = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + q0;
+        bulk_load(sm.nlse2[qb], P.lse2 + off, BQ * 4, &sm.q_full[qb]);
+        bulk_load(sm.ndelta[qb], P.delta + off, BQ * 4, &sm.q_full[qb]);
         ++nq_issued;
         if (t >= 1 && !mbar_wait(&sm.do_empty, (t - 1) & 1, abort, P.status)) break;
-        mbar_arrive_expect_tx(&sm.do_full, BQ * DH * 2 + 2 * BQ * 4);
+        mbar_arrive_expect_tx(&sm.do_full, BQ * DH * 2);
         for (int c = 0; c < DH / 64; ++c)
           tma_load_5d(sm.dO + c * BQ * 64, &P.tm_do, &sm.do_full, c * 64, h, s, q0, b);
-        const long long off = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + q0;
-        bulk_load(sm.lse2, P.lse2 + off, BQ * 4, &sm.do_full);
-        bulk_load(sm.delta, P.delta + off, BQ * 4, &sm.do_full);
         ++ndo_issued;
       }
       // every copy this thread started lands before the CTA may exit
@@ -170,12 +189,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       constexpr uint32_t idKV = idesc_bf16(128, DH, 0, 1);  // dV, dK: A in TMEM, B = dO / Q MN-major
       constexpr uint32_t idQ = idesc_bf16(128, DH, 1, 1);   // dQ: A = dS (dS^T tile MN-major), B = K MN-major
       const uint32_t ka = smem_u32(sm.k), va = smem_u32(sm.v), da = smem_u32(sm.dO), dsa = smem_u32(sm.ds);
+      // S'^T / dP'^T: accumulated from the first k-step onto the pre-filled region
       auto issue_sp = [&](uint32_t aa, uint32_t ba, uint32_t col) {
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
           const uint64_t ad = sdesc_sw128(aa + (kk >> 2) * (BK * 128) + (kk & 3) * 32, 16, 1024);
           const uint64_t bd = sdesc_sw128(ba + (kk >> 2) * (BQ * 128) + (kk & 3) * 32, 16, 1024);
-          tc_mma_ss(tmem + col, ad, bd, idSP, kk > 0 ? 1u : 0u);
+          tc_mma_ss(tmem + col, ad, bd, idSP, 1u);
         }
       };
       // dV (a_col = P^T) or dK (a_col = dS^T) += A * B over query k-steps [k0, k0+2);
@@ -187,12 +207,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
           tc_mma_ts(tmem + d_col, tmem + a_col + kk * 8, bd, idKV, (acc || kk > 0) ? 1u : 0u);
         }
       };
-      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.q_full[0], 0, abort, P.status);
+      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.q_full[0], 0, abort, P.status) &&
+                mbar_wait(&sm.s_init, 0, abort, P.status);
       if (ok) {
         tc_fence_after();
         issue_sp(ka, smem_u32(sm.q[0]), col_r(0));
         tc_commit(&sm.s_full);
-        ok = mbar_wait(&sm.do_full, 0, abort, P.status);
+        ok = mbar_wait(&sm.do_full, 0, abort, P.status) && mbar_wait(&sm.dp_init, 0, abort, P.status);
         if (ok) {
           tc_fence_after();
           issue_sp(va, da, col_r(1));
@@ -211,6 +232,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         if (!ok) break;
         tc_commit(&sm.do_empty);
         tc_commit(&sm.q_empty[p]);
+        tc_commit(&sm.dk_done);  // R[p^1] free for the S'^T(t+1) pre-fill
         // dQ(t) = dS K into R[p] (after dV(t) read P^T there)
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
@@ -221,12 +243,16 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         tc_commit(&sm.dq_full);
         if (t + 1 < T) {
           // S^T(t+1) into R[p^1]: dK(t) has read dS^T(t) from it
-          if (!mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status)) { ok = false; break; }
+          if (!mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status) ||
+              !mbar_wait(&sm.s_init, (t + 1) & 1, abort, P.status)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           issue_sp(ka, smem_u32(sm.q[p ^ 1]), col_r(p ^ 1));
           tc_commit(&sm.s_full);
-          // dP^T(t+1) into R[p]: dQ(t) must have been read out, dO(t+1) loaded
-          if (!mbar_wait(&sm.dq_free, t & 1, abort, P.status) ||
+          // dP^T(t+1) into R[p]: dQ(t) read out and R[p] pre-filled, dO(t+1) loaded
+          if (!mbar_wait(&sm.dp_init, (t + 1) & 1, abort, P.status) ||
               !mbar_wait(&sm.do_full, (t + 1) & 1, abort, P.status)) {
             ok = false;
             break;
@@ -253,8 +279,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       const int p = t & 1;
       const int q0 = (i_lo + t % nq) * BQ;
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status) &&
-                                       mbar_wait(&sm.dp_full, t & 1, abort, P.status) &&
-                                       mbar_wait(&sm.do_full, t & 1, abort, P.status))) {
+                                       mbar_wait(&sm.dp_full, t & 1, abort, P.status))) {
         ok = false;
         break;
       }
@@ -281,28 +306,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
           for (int e = 0; e < 16; ++e)
             if (!visible(q0 + 16 * c + e, kr, G.Lv, G.window)) sr[e] = __float_as_uint(-INFINITY);
         }
-        // sm.lse2 / sm.delta hold -lse*log2(e) and -delta (see sfa_bwd_prep.cu)
-        const float4* l2 = reinterpret_cast<const float4*>(sm.lse2 + 16 * c);
-        const float4* dl = reinterpret_cast<const float4*>(sm.delta + 16 * c);
+        // S'^T and dP'^T already carry -lse2/c2 and -delta (pre-filled accumulators)
         uint32_t pp[8], dd[8];
 #pragma unroll
-        for (int c4 = 0; c4 < 4; ++c4) {
-          const float4 lv = l2[c4], dv = dl[c4];
-#pragma unroll
-          for (int hp = 0; hp < 2; ++hp) {
-            const int e = 4 * c4 + 2 * hp;
-            float x0, x1;
-            f2unpack(ffma2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2,
-                           hp ? f2pack(lv.z, lv.w) : f2pack(lv.x, lv.y)),
-                     x0, x1);
-            const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-            const uint64_t dpd = fadd2(f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1])),
-                                       hp ? f2pack(dv.z, dv.w) : f2pack(dv.x, dv.y));
-            float d0, d1;
-            f2unpack(fmul2(f2pack(p0, p1), dpd), d0, d1);
-            pp[e >> 1] = cvt_bf16x2(p0, p1);
-            dd[e >> 1] = cvt_bf16x2(d0, d1);
-          }
+        for (int e = 0; e < 16; e += 2) {
+          float x0, x1;
+          f2unpack(fmul2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2), x0, x1);
+          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+          float d0, d1;
+          f2unpack(fmul2(f2pack(p0, p1), f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1]))), d0, d1);
+          pp[e >> 1] = cvt_bf16x2(p0, p1);
+          dd[e >> 1] = cvt_bf16x2(d0, d1);
         }
         tmem_st8(tl + col_r(p) + 8 * c, pp);
         tmem_st8(tl + col_r(p ^ 1) + 8 * c, dd);
@@ -349,18 +363,58 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       }
     }
   } else {
-    // ------------------------------------------------------------ dQ flush
-    // TMEM lane = query row q0 + 32*q4 + lane; this warp's 64 head-dim columns leave
-    // TMEM first, then two 32-column rounds are staged (128-byte swizzle) and added
-    // into the fp32 accumulator by TMA reduce.
+    // ------------------------------------------------------------ dQ flush, pre-fills
+    // Pre-fill: every lane of this warp's quadrant gets the same values in columns
+    // [64*dhalf, +64) of a region: -lse2/c2 of the next query tile before its S^T
+    // MMA, -delta before its dP^T MMA.
+    // dQ: TMEM lane = query row q0 + 32*q4 + lane; this warp's 64 head-dim columns
+    // leave TMEM first, then two 32-column rounds are staged (128-byte swizzle) and
+    // added into the fp32 accumulator by TMA reduce.
     const int dhalf = (warp - 6) >> 2;
     const int q4 = warp & 3;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     float* stage = sm.dqs[warp - 6];
-    bool ok = true;
+    const float inv_c2 = 1.f / P.scale_log2;
+    auto prefill = [&](uint32_t col, const float* src, float mul) {
+#pragma unroll 1
+      for (int h4 = 0; h4 < 4; ++h4) {
+        const float4* s4 = reinterpret_cast<const float4*>(src + 64 * dhalf + 16 * h4);
+        uint32_t w[16];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float4 x = s4[i];
+          w[4 * i] = __float_as_uint(x.x * mul);
+          w[4 * i + 1] = __float_as_uint(x.y * mul);
+          w[4 * i + 2] = __float_as_uint(x.z * mul);
+          w[4 * i + 3] = __float_as_uint(x.w * mul);
+        }
+        tmem_st16(tl + col + 64 * dhalf + 16 * h4, w);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+    };
+    // tile 0: S'^T(0) region R0, dP'^T(0) region R1
+    bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.q_full[0], 0, abort, P.status));
+    if (ok) {
+      prefill(col_r(0), sm.nlse2[0], inv_c2);
+      mbar_arrive(&sm.s_init);
+      prefill(col_r(1), sm.ndelta[0], 1.f);
+      mbar_arrive(&sm.dp_init);
+    }
     for (int t = 0; ok && t < T; ++t) {
       const int p = t & 1;
       const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
+      if (t + 1 < T) {
+        // R[p^1] for S'^T(t+1): dK(t) has read dS^T(t) there; row terms of tile t+1 loaded
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.dk_done, t & 1, abort, P.status) &&
+                                         mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        prefill(col_r(p ^ 1), sm.nlse2[p ^ 1], inv_c2);
+        mbar_arrive(&sm.s_init);
+      }
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) {
         ok = false;
         break;
@@ -370,8 +424,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       tmem_ld32(tl + col_r(p) + 64 * dhalf, v);
       tmem_ld32(tl + col_r(p) + 64 * dhalf + 32, v + 32);
       tmem_ld_wait();
-      tc_fence_before();
-      mbar_arrive(&sm.dq_free);  // the MMA may now overwrite these columns
+      if (t + 1 < T) {
+        // dQ(t) is out of R[p]: pre-fill it for dP'^T(t+1)
+        prefill(col_r(p), sm.ndelta[p ^ 1], 1.f);
+        mbar_arrive(&sm.dp_init);
+      }
 #pragma unroll
       for (int r2 = 0; r2 < 2; ++r2) {
         // the previous reduce from this warp's buffer must have read it
@@ -421,7 +478,7 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   p.scale = scale;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.status = status;
-  const int smem = (int)sizeof(Smem) + 1024;
+  const int smem = kSmemBytes;
   cudaError_t e = cudaFuncSetAttribute(bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.ns * g.B);
