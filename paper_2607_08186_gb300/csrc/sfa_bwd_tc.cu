@@ -6,10 +6,11 @@
 // tiles that can see tile j (causal: query tiles at or after the key tile; LOCAL:
 // also within the window).  Every GEMM is a 128 x 128 x 16k tcgen05 MMA (N = 128
 // runs at full tensor rate; N = 64 does not):
-//   S'^T = K Q^T - lse2/c2,  dP'^T = V dO^T - delta
+//   S'^T = K Q^T - lse2/c2 (-inf on masked pairs),  dP'^T = V dO^T - delta
 //                                       SS: A = K / V (K-major), B = Q / dO (K-major),
 //                                       accumulated onto TMEM pre-filled with the
-//                                       per-query terms (c2 = scale*log2e, lse2 = lse*log2e)
+//                                       per-query terms and the mask (c2 = scale*log2e,
+//                                       lse2 = lse*log2e)
 //   P^T  = exp2(c2 S'^T),  dS^T = P^T dP'^T              (softmax; packed f32x2
 //                                       arithmetic, exp2 on the SFU, no shared memory)
 //   dV  += P^T dO,  dK += dS^T Q        TS: A = P^T / dS^T packed bf16 in TMEM
@@ -277,46 +278,45 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     bool ok = true;
     for (int t = 0; t < T; ++t) {
       const int p = t & 1;
-      const int q0 = (i_lo + t % nq) * BQ;
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status) &&
                                        mbar_wait(&sm.dp_full, t & 1, abort, P.status))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const bool need_mask = (q0 < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (q0 + BQ > G.Lv);
       // eight chunks of 16 query columns; the TMEM loads of chunk c+1 are in flight
       // while chunk c is computed.  Chunk c packs into columns [8c, 8c+8), which hold
       // data of chunks this thread has already read (and no chunk still to be loaded).
+      // The chunk loop stays rolled, two chunks per iteration so that the double
+      // buffer is indexed statically (measured as fast as fully unrolled, with an
+      // eighth of the code).
       const uint64_t c2x2 = f2pack(c2, c2);
       uint32_t sbuf[2][16], dbuf[2][16];
-      tmem_ld16(tl + col_r(p), sbuf[0]);
-      tmem_ld16(tl + col_r(p ^ 1), dbuf[0]);
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint32_t* sr = sbuf[c & 1];
-        uint32_t* dr = dbuf[c & 1];
+      auto chunk = [&](int c, uint32_t* sr, uint32_t* dr, uint32_t* sn, uint32_t* dn) {
         tmem_ld_wait();  // chunk c has landed (the only loads in flight)
         if (c + 1 < 8) {
-          tmem_ld16(tl + col_r(p) + 16 * (c + 1), sbuf[(c + 1) & 1]);
-          tmem_ld16(tl + col_r(p ^ 1) + 16 * (c + 1), dbuf[(c + 1) & 1]);
+          tmem_ld16(tl + col_r(p) + 16 * (c + 1), sn);
+          tmem_ld16(tl + col_r(p ^ 1) + 16 * (c + 1), dn);
         }
-        if (need_mask) {
+        // S'^T and dP'^T already carry -lse2/c2 (or -inf where masked) and -delta
+        // (pre-filled accumulators).
+        // One step over all 16 elements at a time, so the 8 independent pairs hide each
+        // other's latency (written per element pair, the chains issue one after another).
+        float x[16], pv[16], dv[16];
 #pragma unroll
-          for (int e = 0; e < 16; ++e)
-            if (!visible(q0 + 16 * c + e, kr, G.Lv, G.window)) sr[e] = __float_as_uint(-INFINITY);
-        }
-        // S'^T and dP'^T already carry -lse2/c2 and -delta (pre-filled accumulators)
+        for (int e = 0; e < 16; e += 2)
+          f2unpack(fmul2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2), x[e], x[e + 1]);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) pv[e] = ex2_approx(x[e]);
+#pragma unroll
+        for (int e = 0; e < 16; e += 2)
+          f2unpack(fmul2(f2pack(pv[e], pv[e + 1]), f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1]))),
+                   dv[e], dv[e + 1]);
         uint32_t pp[8], dd[8];
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
-          float x0, x1;
-          f2unpack(fmul2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2), x0, x1);
-          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-          float d0, d1;
-          f2unpack(fmul2(f2pack(p0, p1), f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1]))), d0, d1);
-          pp[e >> 1] = cvt_bf16x2(p0, p1);
-          dd[e >> 1] = cvt_bf16x2(d0, d1);
+          pp[e >> 1] = cvt_bf16x2(pv[e], pv[e + 1]);
+          dd[e >> 1] = cvt_bf16x2(dv[e], dv[e + 1]);
         }
         tmem_st8(tl + col_r(p) + 8 * c, pp);
         tmem_st8(tl + col_r(p ^ 1) + 8 * c, dd);
@@ -326,14 +326,19 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         for (int k = 0; k < 2; ++k)
           *reinterpret_cast<uint4*>(blk + (((2 * (c & 3) + k) ^ (row & 7)) << 4)) =
               make_uint4(dd[4 * k], dd[4 * k + 1], dd[4 * k + 2], dd[4 * k + 3]);
-        if (c & 1) {
-          // query quarter c/2 packed: its dV / dK k-steps may start; after the last
-          // quarter the whole dS^T tile is also in shared memory for dQ(t)
-          if (c == 7) fence_async_smem();
-          tmem_st_wait();
-          tc_fence_before();
-          mbar_arrive(&sm.p_part[c >> 1]);
-        }
+      };
+      tmem_ld16(tl + col_r(p), sbuf[0]);
+      tmem_ld16(tl + col_r(p ^ 1), dbuf[0]);
+#pragma unroll 1
+      for (int c = 0; c < 8; c += 2) {
+        chunk(c, sbuf[0], dbuf[0], sbuf[1], dbuf[1]);
+        chunk(c + 1, sbuf[1], dbuf[1], sbuf[0], dbuf[0]);
+        // query quarter c/2 packed: its dV / dK k-steps may start; after the last
+        // quarter the whole dS^T tile is also in shared memory for dQ(t)
+        if (c == 6) fence_async_smem();
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&sm.p_part[c >> 1]);
       }
     }
     // epilogue: this key row of dV, then of dK (scaled)
@@ -364,9 +369,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     }
   } else {
     // ------------------------------------------------------------ dQ flush, pre-fills
-    // Pre-fill: every lane of this warp's quadrant gets the same values in columns
-    // [64*dhalf, +64) of a region: -lse2/c2 of the next query tile before its S^T
-    // MMA, -delta before its dP^T MMA.
+    // Pre-fill, columns [64*dhalf, +64) of a region, this warp's TMEM lanes (key rows):
+    // -lse2/c2 of the next query tile before its S^T MMA, with -inf where the key row
+    // does not see the query (the mask: exp2 then gives P = 0 whatever the MMA adds);
+    // -delta before its dP^T MMA.
     // dQ: TMEM lane = query row q0 + 32*q4 + lane; this warp's 64 head-dim columns
     // leave TMEM first, then two 32-column rounds are staged (128-byte swizzle) and
     // added into the fp32 accumulator by TMA reduce.
@@ -375,7 +381,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     float* stage = sm.dqs[warp - 6];
     const float inv_c2 = 1.f / P.scale_log2;
-    auto prefill = [&](uint32_t col, const float* src, float mul) {
+    const int kr = n0 + q4 * 32 + lane;  // key row of this thread's TMEM lane
+    // qm >= 0: query tile start of an S'^T pre-fill (masked where needed); -1: dP'^T
+    auto prefill = [&](uint32_t col, const float* src, float mul, int qm) {
+      const bool mask = qm >= 0 && ((qm < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (qm + BQ > G.Lv));
 #pragma unroll 1
       for (int h4 = 0; h4 < 4; ++h4) {
         const float4* s4 = reinterpret_cast<const float4*>(src + 64 * dhalf + 16 * h4);
@@ -388,6 +397,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
           w[4 * i + 2] = __float_as_uint(x.z * mul);
           w[4 * i + 3] = __float_as_uint(x.w * mul);
         }
+        if (mask) {
+          const int qc = qm + 64 * dhalf + 16 * h4;
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (!visible(qc + i, kr, G.Lv, G.window)) w[i] = __float_as_uint(-INFINITY);
+        }
         tmem_st16(tl + col + 64 * dhalf + 16 * h4, w);
       }
       tmem_st_wait();
@@ -396,9 +411,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     // tile 0: S'^T(0) region R0, dP'^T(0) region R1
     bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.q_full[0], 0, abort, P.status));
     if (ok) {
-      prefill(col_r(0), sm.nlse2[0], inv_c2);
+      prefill(col_r(0), sm.nlse2[0], inv_c2, i_lo * BQ);
       mbar_arrive(&sm.s_init);
-      prefill(col_r(1), sm.ndelta[0], 1.f);
+      prefill(col_r(1), sm.ndelta[0], 1.f, -1);
       mbar_arrive(&sm.dp_init);
     }
     for (int t = 0; ok && t < T; ++t) {
@@ -412,7 +427,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
           break;
         }
         tc_fence_after();
-        prefill(col_r(p ^ 1), sm.nlse2[p ^ 1], inv_c2);
+        prefill(col_r(p ^ 1), sm.nlse2[p ^ 1], inv_c2, (i_lo + (t + 1) % nq) * BQ);
         mbar_arrive(&sm.s_init);
       }
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) {
@@ -426,7 +441,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       tmem_ld_wait();
       if (t + 1 < T) {
         // dQ(t) is out of R[p]: pre-fill it for dP'^T(t+1)
-        prefill(col_r(p), sm.ndelta[p ^ 1], 1.f);
+        prefill(col_r(p), sm.ndelta[p ^ 1], 1.f, -1);
         mbar_arrive(&sm.dp_init);
       }
 #pragma unroll
