@@ -382,53 +382,81 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     float* stage = sm.dqs[warp - 6];
     const float inv_c2 = 1.f / P.scale_log2;
     const int kr = n0 + q4 * 32 + lane;  // key row of this thread's TMEM lane
-    // qm >= 0: query tile start of an S'^T pre-fill (masked where needed); -1: dP'^T
-    auto prefill = [&](uint32_t col, const float* src, float mul, int qm) {
-      const bool mask = qm >= 0 && ((qm < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (qm + BQ > G.Lv));
-#pragma unroll 1
-      for (int h4 = 0; h4 < 4; ++h4) {
-        const float4* s4 = reinterpret_cast<const float4*>(src + 64 * dhalf + 16 * h4);
-        uint32_t w[16];
+    // Pre-fill values for this warp's 64 columns are read from shared memory and
+    // masked before the region is free (those loads would otherwise queue behind the
+    // MMAs' operand reads on the critical path); only the TMEM stores follow the wait.
+    // S'^T of the query tile starting at qm: -lse2/c2, -inf where not visible.
+    auto s_values = [&](uint32_t* w, const float* src, int qm) {
+      const float4* s4 = reinterpret_cast<const float4*>(src + 64 * dhalf);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float4 x = s4[i];
-          w[4 * i] = __float_as_uint(x.x * mul);
-          w[4 * i + 1] = __float_as_uint(x.y * mul);
-          w[4 * i + 2] = __float_as_uint(x.z * mul);
-          w[4 * i + 3] = __float_as_uint(x.w * mul);
-        }
-        if (mask) {
-          const int qc = qm + 64 * dhalf + 16 * h4;
-#pragma unroll
-          for (int i = 0; i < 16; ++i)
-            if (!visible(qc + i, kr, G.Lv, G.window)) w[i] = __float_as_uint(-INFINITY);
-        }
-        tmem_st16(tl + col + 64 * dhalf + 16 * h4, w);
+      for (int i = 0; i < 16; ++i) {
+        const float4 x = s4[i];
+        w[4 * i] = __float_as_uint(x.x * inv_c2);
+        w[4 * i + 1] = __float_as_uint(x.y * inv_c2);
+        w[4 * i + 2] = __float_as_uint(x.z * inv_c2);
+        w[4 * i + 3] = __float_as_uint(x.w * inv_c2);
       }
+      if ((qm < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (qm + BQ > G.Lv)) {
+        // key row kr sees the queries q in [kr, vis_hi): causal, inside the sequence,
+        // and for LOCAL inside the window (an empty range when kr itself is past Lv)
+        const long long lim = G.window > 0 ? min((long long)G.Lv, (long long)kr + G.window) : (long long)G.Lv;
+        const int vis_hi = kr < G.Lv ? (int)lim : kr;
+        const int qb = qm + 64 * dhalf;
+#pragma unroll
+        for (int i = 0; i < 64; ++i)
+          if (qb + i < kr || qb + i >= vis_hi) w[i] = __float_as_uint(-INFINITY);
+      }
+    };
+    auto d_values = [&](uint32_t* w, const float* src) {  // dP'^T: -delta
+      const uint4* s4 = reinterpret_cast<const uint4*>(src + 64 * dhalf);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const uint4 x = s4[i];
+        w[4 * i] = x.x;
+        w[4 * i + 1] = x.y;
+        w[4 * i + 2] = x.z;
+        w[4 * i + 3] = x.w;
+      }
+    };
+    auto store64 = [&](uint32_t col, const uint32_t* w) {
+      tmem_st32(tl + col + 64 * dhalf, w);
+      tmem_st32(tl + col + 64 * dhalf + 32, w + 32);
+    };
+    auto publish = [&](uint64_t* bar) {  // stores landed, then signal the MMA thread
       tmem_st_wait();
       tc_fence_before();
+      mbar_arrive(bar);
     };
     // tile 0: S'^T(0) region R0, dP'^T(0) region R1
     bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.q_full[0], 0, abort, P.status));
     if (ok) {
-      prefill(col_r(0), sm.nlse2[0], inv_c2, i_lo * BQ);
-      mbar_arrive(&sm.s_init);
-      prefill(col_r(1), sm.ndelta[0], 1.f, -1);
-      mbar_arrive(&sm.dp_init);
+      uint32_t w[64];
+      s_values(w, sm.nlse2[0], i_lo * BQ);
+      store64(col_r(0), w);
+      publish(&sm.s_init);
+      d_values(w, sm.ndelta[0]);
+      store64(col_r(1), w);
+      publish(&sm.dp_init);
     }
     for (int t = 0; ok && t < T; ++t) {
       const int p = t & 1;
       const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
-      if (t + 1 < T) {
-        // R[p^1] for S'^T(t+1): dK(t) has read dS^T(t) there; row terms of tile t+1 loaded
-        if (!__all_sync(0xffffffffu, mbar_wait(&sm.dk_done, t & 1, abort, P.status) &&
-                                         mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status))) {
+      const bool next = t + 1 < T;
+      if (next) {
+        // R[p^1] for S'^T(t+1): row terms of tile t+1 loaded; dK(t) has read dS^T(t) there
+        uint32_t w[64];
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status))) {
+          ok = false;
+          break;
+        }
+        s_values(w, sm.nlse2[p ^ 1], (i_lo + (t + 1) % nq) * BQ);
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.dk_done, t & 1, abort, P.status))) {
           ok = false;
           break;
         }
         tc_fence_after();
-        prefill(col_r(p ^ 1), sm.nlse2[p ^ 1], inv_c2, (i_lo + (t + 1) % nq) * BQ);
-        mbar_arrive(&sm.s_init);
+        store64(col_r(p ^ 1), w);
+        publish(&sm.s_init);
       }
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full, t & 1, abort, P.status))) {
         ok = false;
@@ -439,10 +467,23 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       tmem_ld32(tl + col_r(p) + 64 * dhalf, v);
       tmem_ld32(tl + col_r(p) + 64 * dhalf + 32, v + 32);
       tmem_ld_wait();
-      if (t + 1 < T) {
-        // dQ(t) is out of R[p]: pre-fill it for dP'^T(t+1)
-        prefill(col_r(p), sm.ndelta[p ^ 1], 1.f, -1);
-        mbar_arrive(&sm.dp_init);
+      if (next) {
+        // dQ(t) is out of R[p]: pre-fill it for dP'^T(t+1), 16 columns at a time
+#pragma unroll 1
+        for (int h4 = 0; h4 < 4; ++h4) {
+          const uint4* s4 = reinterpret_cast<const uint4*>(sm.ndelta[p ^ 1] + 64 * dhalf + 16 * h4);
+          uint32_t w[16];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const uint4 x = s4[i];
+            w[4 * i] = x.x;
+            w[4 * i + 1] = x.y;
+            w[4 * i + 2] = x.z;
+            w[4 * i + 3] = x.w;
+          }
+          tmem_st16(tl + col_r(p) + 64 * dhalf + 16 * h4, w);
+        }
+        publish(&sm.dp_init);
       }
 #pragma unroll
       for (int r2 = 0; r2 < 2; ++r2) {
