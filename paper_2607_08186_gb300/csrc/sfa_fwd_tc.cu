@@ -151,13 +151,20 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
         tc_fence_after();
         return true;
       };
+      // Operand descriptors are encoded once; k-step kk adds its byte offset / 16 to the
+      // 64-bit descriptor (the address field; shared addresses stay below 256 KB), which
+      // keeps the instructions between consecutive MMAs (and so the issue gaps) small.
+      static_assert(BM == 128 && BN == 128 && NST == 2 && NG == 2, "descriptor bases below");
+      const uint64_t qK0 = sdesc_sw128(smem_u32(sm.q[0]), 16, 1024), qK1 = sdesc_sw128(smem_u32(sm.q[1]), 16, 1024);
+      const uint64_t kK0 = sdesc_sw128(smem_u32(sm.k[0]), 16, 1024), kK1 = sdesc_sw128(smem_u32(sm.k[1]), 16, 1024);
+      const uint64_t vM0 = sdesc_sw128(smem_u32(sm.v[0]), BN * 128, 1024),
+                     vM1 = sdesc_sw128(smem_u32(sm.v[1]), BN * 128, 1024);
       auto issue_s = [&](int g, int j) {
-        const uint32_t qa = smem_u32(sm.q[g]), ka = smem_u32(sm.k[(j - n_lo) % NST]);
+        const uint64_t qd = g ? qK1 : qK0, kd = ((j - n_lo) & 1) ? kK1 : kK0;
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint64_t ad = sdesc_sw128(qa + (kk >> 2) * (BM * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd = sdesc_sw128(ka + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
-          tc_mma_ss(tmem + g * 128, ad, bd, idS, kk > 0 ? 1u : 0u);
+          const uint64_t off = (uint64_t)((kk >> 2) * (128 * 128 / 16) + (kk & 3) * 2);
+          tc_mma_ss(tmem + g * 128, qd + off, kd + off, idS, kk > 0 ? 1u : 0u);
         }
         tc_commit(&sm.s_full[g]);
       };
@@ -165,12 +172,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
         if (!mbar_wait(&sm.p_full[g], ps[g] & 1, abort, P.status)) return false;
         ++ps[g];
         tc_fence_after();
-        const uint32_t va = smem_u32(sm.v[(j - n_lo) % NST]);
+        const uint64_t vd = ((j - n_lo) & 1) ? vM1 : vM0;
 #pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, BN * 128, 1024);
-          tc_mma_ts(tmem + 256 + g * DH, tmem + g * 128 + kk * 8, bd, idO, (j > lo[g] || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < BN / 16; ++kk)
+          tc_mma_ts(tmem + 256 + g * DH, tmem + g * 128 + kk * 8, vd + (uint64_t)(kk * 16 * 128 / 16), idO,
+                    (j > lo[g] || kk > 0) ? 1u : 0u);
         return true;
       };
       if (ok && n_hi >= n_lo && wait_kv(n_lo)) {
