@@ -11,8 +11,9 @@
 //                                       accumulated onto TMEM pre-filled with the
 //                                       per-query terms and the mask (c2 = scale*log2e,
 //                                       lse2 = lse*log2e)
-//   P^T  = exp2(c2 S'^T),  dS^T = P^T dP'^T              (softmax; packed f32x2
-//                                       arithmetic, exp2 on the SFU, no shared memory)
+//   P^T  = exp2(c2 S'^T)      (softmax phase A: needs S'^T only)
+//   dS^T = P^T dP'^T          (phase B: P^T read back as the bf16 the dV MMA uses)
+//                             packed f32x2 arithmetic, exp2 on the SFU
 //   dV  += P^T dO,  dK += dS^T Q        TS: A = P^T / dS^T packed bf16 in TMEM
 //   dQ   = dS K                         SS: A = dS^T tile in smem read MN-major,
 //                                           B = K read MN-major; TMEM lane = query row
@@ -24,10 +25,12 @@
 // TMEM: two 128-column regions R0, R1 swap roles with the tile parity p:
 //   S^T(t) in R[p] (P^T packed bf16 over its first 64 columns, then dQ(t)),
 //   dP^T(t) in R[p^1] (dS^T packed bf16 over its first 64 columns);  dV at 256, dK at 384.
-// MMA issue order:  for each quarter u of the query columns: wait P(t) quarter u |
-//                   dV(t), dK(t) k-steps of quarter u;  then dQ(t) | wait R[p^1]
-//                   pre-filled | S(t+1) | wait dQ(t) read out and R[p] pre-filled | dP(t+1)
-// so three quarters of dV(t), dK(t) run under the softmax of the later columns.
+// MMA issue order:  for each quarter u of the query columns: wait P^T(t) quarter u |
+//                   dV(t) k-steps of u;  then per quarter: wait dS^T(t) quarter u | dK(t)
+//                   k-steps of u;  dQ(t) | wait R[p^1] pre-filled | S(t+1) | wait dQ(t)
+//                   read out and R[p] pre-filled | dP(t+1)
+// Phase A of tile t+1 needs only S'^T(t+1), so it overlaps the dQ(t) read-out, the
+// dP(t+1) pre-fill and the dP(t+1) MMA; dV / dK k-steps run under the later quarters.
 // The pre-fills (every TMEM lane gets the same 128 per-query values) are written
 // by the dQ warps: R[p^1] once dK(t) has read dS^T(t) (under dQ(t)), R[p] right
 // after they have read dQ(t) out of it.
@@ -62,7 +65,7 @@ struct Smem {
   float dqs[8][32 * 32];  // per dQ warp: [32 query rows][32 head-dim] fp32, 128-byte swizzle
   float nlse2[2][BQ];     // -lse*log2(e) of the query tile in q[i], loaded with it
   float ndelta[2][BQ];    // -delta of the query tile in q[i], loaded with it
-  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, p_part[4], dq_full, s_init,
+  uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, pa_part[4], pb_part[4], dq_full, s_init,
       dp_init, dk_done, kv_done, drain;
   uint32_t tmem_base;
   int abort;
@@ -127,7 +130,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     mbar_init(&sm.do_empty, 1);
     mbar_init(&sm.s_full, 1);
     mbar_init(&sm.dp_full, 1);
-    for (int i = 0; i < 4; ++i) mbar_init(&sm.p_part[i], 128);
+    for (int i = 0; i < 4; ++i) {
+      mbar_init(&sm.pa_part[i], 128);
+      mbar_init(&sm.pb_part[i], 128);
+    }
     mbar_init(&sm.dq_full, 1);
     mbar_init(&sm.s_init, 256);
     mbar_init(&sm.dp_init, 256);
@@ -233,16 +239,21 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         const int p = t & 1;
         const uint64_t qM = p ? qM1 : qM0;
         for (int u = 0; u < 4; ++u) {
-          if (!mbar_wait(&sm.p_part[u], t & 1, abort, P.status)) { ok = false; break; }
+          if (!mbar_wait(&sm.pa_part[u], t & 1, abort, P.status)) { ok = false; break; }
           tc_fence_after();
           issue_kv(col_r(p), doM, COL_DV, t > 0, 2 * u);       // reads P^T(t) and dO(t)
-          issue_kv(col_r(p ^ 1), qM, COL_DK, t > 0, 2 * u);    // reads dS^T(t) and Q(t)
         }
         if (!ok) break;
         tc_commit(&sm.do_empty);
+        for (int u = 0; u < 4; ++u) {
+          if (!mbar_wait(&sm.pb_part[u], t & 1, abort, P.status)) { ok = false; break; }
+          tc_fence_after();
+          issue_kv(col_r(p ^ 1), qM, COL_DK, t > 0, 2 * u);    // reads dS^T(t) and Q(t)
+        }
+        if (!ok) break;
         tc_commit(&sm.q_empty[p]);
         tc_commit(&sm.dk_done);  // R[p^1] free for the S'^T(t+1) pre-fill
-        // dQ(t) = dS K into R[p] (after dV(t) read P^T there)
+        // dQ(t) = dS K into R[p] (after dV(t) and phase B(t) read P^T there)
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk)
           tc_mma_ss(tmem + col_r(p), dsM + moff(kk), kM + moff(kk), idQ, kk > 0 ? 1u : 0u);
@@ -283,65 +294,89 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     bool ok = true;
     for (int t = 0; t < T; ++t) {
       const int p = t & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status) &&
-                                       mbar_wait(&sm.dp_full, t & 1, abort, P.status))) {
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.s_full, t & 1, abort, P.status))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      // eight chunks of 16 query columns; the TMEM loads of chunk c+1 are in flight
-      // while chunk c is computed.  Chunk c packs into columns [8c, 8c+8), which hold
-      // data of chunks this thread has already read (and no chunk still to be loaded).
-      // Fully unrolled (rolled, the loop ran at ~0.55x the speed).
+      // Eight chunks of 16 query columns per phase; the TMEM loads of chunk c+1 are in
+      // flight while chunk c is computed.  Chunk c packs into columns [8c, 8c+8), which
+      // hold data this thread has already read.  Each quarter is published with its
+      // stores landed, so the MMAs of that quarter may start.
       const uint64_t c2x2 = f2pack(c2, c2);
-      uint32_t sbuf[2][16], dbuf[2][16];
-      auto chunk = [&](int c, uint32_t* sr, uint32_t* dr, uint32_t* sn, uint32_t* dn) {
-        tmem_ld_wait();  // chunk c has landed (the only loads in flight)
-        if (c + 1 < 8) {
-          tmem_ld16(tl + col_r(p) + 16 * (c + 1), sn);
-          tmem_ld16(tl + col_r(p ^ 1) + 16 * (c + 1), dn);
+      // ---- phase A: P^T = exp2(c2 S'^T), S'^T already carrying -lse2/c2 (or -inf
+      // where masked), packed bf16 into R[p]
+      {
+        uint32_t sbuf[2][16];
+        auto chunk_a = [&](int c, uint32_t* sr, uint32_t* sn) {
+          tmem_ld_wait();
+          if (c + 1 < 8) tmem_ld16(tl + col_r(p) + 16 * (c + 1), sn);
+          float x[16], pv[16];
+#pragma unroll
+          for (int e = 0; e < 16; e += 2)
+            f2unpack(fmul2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2), x[e], x[e + 1]);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) pv[e] = ex2_approx(x[e]);
+          uint32_t pp[8];
+#pragma unroll
+          for (int e = 0; e < 16; e += 2) pp[e >> 1] = cvt_bf16x2(pv[e], pv[e + 1]);
+          tmem_st8(tl + col_r(p) + 8 * c, pp);
+        };
+        tmem_ld16(tl + col_r(p), sbuf[0]);
+#pragma unroll
+        for (int c = 0; c < 8; c += 2) {
+          chunk_a(c, sbuf[0], sbuf[1]);
+          chunk_a(c + 1, sbuf[1], sbuf[0]);
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(&sm.pa_part[c >> 1]);
         }
-        // S'^T and dP'^T already carry -lse2/c2 (or -inf where masked) and -delta
-        // (pre-filled accumulators).
-        // One step over all 16 elements at a time, so the 8 independent pairs hide each
-        // other's latency (written per element pair, the chains issue one after another).
-        float x[16], pv[16], dv[16];
+      }
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.dp_full, t & 1, abort, P.status))) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      // ---- phase B: dS^T = P^T dP'^T (P^T as packed bf16 from R[p], dP'^T already
+      // carrying -delta), packed bf16 into R[p^1] and into shared memory for dQ(t)
+      {
+        uint32_t dbuf[2][16], pbuf[2][8];
+        auto chunk_b = [&](int c, uint32_t* dr, uint32_t* pr, uint32_t* dn, uint32_t* pn) {
+          tmem_ld_wait();
+          if (c + 1 < 8) {
+            tmem_ld16(tl + col_r(p ^ 1) + 16 * (c + 1), dn);
+            tmem_ld8(tl + col_r(p) + 8 * (c + 1), pn);
+          }
+          uint32_t dd[8];
 #pragma unroll
-        for (int e = 0; e < 16; e += 2)
-          f2unpack(fmul2(f2pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), c2x2), x[e], x[e + 1]);
+          for (int e = 0; e < 16; e += 2) {
+            const uint32_t w = pr[e >> 1];  // P of elements e (low half) and e+1 (high half)
+            float d0, d1;
+            f2unpack(fmul2(f2pack(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u)),
+                           f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1]))),
+                     d0, d1);
+            dd[e >> 1] = cvt_bf16x2(d0, d1);
+          }
+          tmem_st8(tl + col_r(p ^ 1) + 8 * c, dd);
+          // dS^T -> shared memory for dQ(t): block c/4, 16-byte chunks 2(c%4), 2(c%4)+1
+          uint8_t* blk = dsrow + (c >> 2) * (BK * 128);
 #pragma unroll
-        for (int e = 0; e < 16; ++e) pv[e] = ex2_approx(x[e]);
+          for (int k = 0; k < 2; ++k)
+            *reinterpret_cast<uint4*>(blk + (((2 * (c & 3) + k) ^ (row & 7)) << 4)) =
+                make_uint4(dd[4 * k], dd[4 * k + 1], dd[4 * k + 2], dd[4 * k + 3]);
+        };
+        tmem_ld16(tl + col_r(p ^ 1), dbuf[0]);
+        tmem_ld8(tl + col_r(p), pbuf[0]);
 #pragma unroll
-        for (int e = 0; e < 16; e += 2)
-          f2unpack(fmul2(f2pack(pv[e], pv[e + 1]), f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1]))),
-                   dv[e], dv[e + 1]);
-        uint32_t pp[8], dd[8];
-#pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          pp[e >> 1] = cvt_bf16x2(pv[e], pv[e + 1]);
-          dd[e >> 1] = cvt_bf16x2(dv[e], dv[e + 1]);
+        for (int c = 0; c < 8; c += 2) {
+          chunk_b(c, dbuf[0], pbuf[0], dbuf[1], pbuf[1]);
+          chunk_b(c + 1, dbuf[1], pbuf[1], dbuf[0], pbuf[0]);
+          // after the last quarter the whole dS^T tile is also in shared memory for dQ(t)
+          if (c == 6) fence_async_smem();
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(&sm.pb_part[c >> 1]);
         }
-        tmem_st8(tl + col_r(p) + 8 * c, pp);
-        tmem_st8(tl + col_r(p ^ 1) + 8 * c, dd);
-        // dS^T -> shared memory for dQ(t): block c/4, 16-byte chunks 2(c%4), 2(c%4)+1
-        uint8_t* blk = dsrow + (c >> 2) * (BK * 128);
-#pragma unroll
-        for (int k = 0; k < 2; ++k)
-          *reinterpret_cast<uint4*>(blk + (((2 * (c & 3) + k) ^ (row & 7)) << 4)) =
-              make_uint4(dd[4 * k], dd[4 * k + 1], dd[4 * k + 2], dd[4 * k + 3]);
-      };
-      tmem_ld16(tl + col_r(p), sbuf[0]);
-      tmem_ld16(tl + col_r(p ^ 1), dbuf[0]);
-#pragma unroll
-      for (int c = 0; c < 8; c += 2) {
-        chunk(c, sbuf[0], dbuf[0], sbuf[1], dbuf[1]);
-        chunk(c + 1, sbuf[1], dbuf[1], sbuf[0], dbuf[0]);
-        // query quarter c/2 packed: its dV / dK k-steps may start; after the last
-        // quarter the whole dS^T tile is also in shared memory for dQ(t)
-        if (c == 6) fence_async_smem();
-        tmem_st_wait();
-        tc_fence_before();
-        mbar_arrive(&sm.p_part[c >> 1]);
       }
     }
     // epilogue: this key row of dV, then of dK (scaled)
