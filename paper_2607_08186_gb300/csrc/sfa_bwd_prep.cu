@@ -14,6 +14,10 @@ namespace hdsfa {
 
 typedef __nv_bfloat16 bf16;
 
+// One warp takes RPW consecutive (b, p, h) rows: DH/8 lanes per row (16 bytes of O and
+// of dO each), 32*8/DH rows side by side, ITER such row groups with every load issued
+// before the first dot product, so each warp keeps several KB in flight.  The warp
+// then zeroes the same rows of the fp32 dQ accumulator (contiguous, 16-byte stores).
 template <int DH>
 __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restrict__ o,
                                                            const bf16* __restrict__ dout,
@@ -21,30 +25,49 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
                                                            float* __restrict__ lse2_t,
                                                            float* __restrict__ delta_t,
                                                            float* __restrict__ dq_acc, SfaGeom g) {
-  const int lane = threadIdx.x & 31;
-  const long long row = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // (b, p, h)
-  if (row >= (long long)g.B * g.nL * g.Hq) return;
-  float acc = 0.f;
-  if (lane < DH / 8) {
-    const uint4 x = *reinterpret_cast<const uint4*>(o + row * DH + lane * 8);
-    const uint4 y = *reinterpret_cast<const uint4*>(dout + row * DH + lane * 8);
-    const bf16* xa = reinterpret_cast<const bf16*>(&x);
-    const bf16* ya = reinterpret_cast<const bf16*>(&y);
+  constexpr int LPR = DH / 8;        // lanes per row
+  constexpr int RPG = 32 / LPR;      // rows per group of the warp
+  constexpr int ITER = 4;            // row groups per warp
+  constexpr int RPW = RPG * ITER;    // rows per warp
+  const int lane = threadIdx.x & 31, sub = lane / LPR, l = lane % LPR;
+  const long long nrows = (long long)g.B * g.nL * g.Hq;
+  const long long row0 = (((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * RPW;
+  if (row0 >= nrows) return;
+  uint4 xo[ITER], xd[ITER];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) acc += __bfloat162float(xa[i]) * __bfloat162float(ya[i]);
+  for (int i = 0; i < ITER; ++i) {
+    const long long row = row0 + i * RPG + sub;
+    if (row < nrows) {
+      xo[i] = *reinterpret_cast<const uint4*>(o + row * DH + l * 8);
+      xd[i] = *reinterpret_cast<const uint4*>(dout + row * DH + l * 8);
+    } else {
+      xo[i] = make_uint4(0, 0, 0, 0);
+      xd[i] = make_uint4(0, 0, 0, 0);
+    }
   }
+  const int Lvp = row_terms_pitch(g.Lv);
 #pragma unroll
-  for (int off = 16; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  float4* dqr = reinterpret_cast<float4*>(dq_acc + row * DH);
-  for (int c = lane; c < DH / 4; c += 32) dqr[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (lane == 0) {
-    const long long h = row % g.Hq, bp = row / g.Hq, p = bp % g.nL, b = bp / g.nL;
-    const int Lvp = row_terms_pitch(g.Lv);
-    const long long s = p % g.ns, r = p / g.ns;
-    const long long t = ((b * g.Hq + h) * g.ns + s) * Lvp + r;
-    delta_t[t] = -acc;
-    lse2_t[t] = -lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
+  for (int i = 0; i < ITER; ++i) {
+    const bf16* xa = reinterpret_cast<const bf16*>(&xo[i]);
+    const bf16* ya = reinterpret_cast<const bf16*>(&xd[i]);
+    float acc = 0.f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc += __bfloat162float(xa[e]) * __bfloat162float(ya[e]);
+#pragma unroll
+    for (int off = LPR / 2; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    const long long row = row0 + i * RPG + sub;
+    if (l == 0 && row < nrows) {
+      const long long h = row % g.Hq, bp = row / g.Hq, p = bp % g.nL, b = bp / g.nL;
+      const long long s = p % g.ns, r = p / g.ns;
+      const long long t = ((b * g.Hq + h) * g.ns + s) * Lvp + r;
+      delta_t[t] = -acc;
+      lse2_t[t] = -lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
+    }
   }
+  // zero dQ accumulator rows [row0, row0 + RPW): RPW * DH floats, contiguous
+  const long long nz = (min(nrows, row0 + RPW) - row0) * DH / 4;
+  float4* dz = reinterpret_cast<float4*>(dq_acc + row0 * DH);
+  for (long long c = lane; c < nz; c += 32) dz[c] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 __global__ void sfa_bwd_pad_kernel(float* __restrict__ lse2_t, float* __restrict__ delta_t, SfaGeom g) {
@@ -75,7 +98,9 @@ cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* ls
                                 float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
                                 cudaStream_t st) {
   const long long rows = (long long)g.B * g.nL * g.Hq;
-  const unsigned blocks = (unsigned)((rows * 32 + 255) / 256);
+  const long long rpw = 4LL * (32 / (Dh / 8));  // rows per warp (ITER * rows per group)
+  const long long warps = (rows + rpw - 1) / rpw;
+  const unsigned blocks = (unsigned)((warps * 32 + 255) / 256);
   if (Dh == 64)
     sfa_bwd_prep_kernel<64><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, lse, lse2_ws,
                                                    delta_ws, dq_ws, g);
