@@ -347,16 +347,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
             tmem_ld16(tl + col_r(p ^ 1) + 16 * (c + 1), dn);
             tmem_ld8(tl + col_r(p) + 8 * (c + 1), pn);
           }
+          // dS pair = bf16(P pair) * bf16(dP' pair) in one packed bf16 multiply: one more
+          // rounding (of dP', relative 2^-9) than an fp32 product rounded to bf16
           uint32_t dd[8];
 #pragma unroll
-          for (int e = 0; e < 16; e += 2) {
-            const uint32_t w = pr[e >> 1];  // P of elements e (low half) and e+1 (high half)
-            float d0, d1;
-            f2unpack(fmul2(f2pack(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u)),
-                           f2pack(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1]))),
-                     d0, d1);
-            dd[e >> 1] = cvt_bf16x2(d0, d1);
-          }
+          for (int e = 0; e < 16; e += 2)
+            dd[e >> 1] = mul_bf16x2(pr[e >> 1], cvt_bf16x2(__uint_as_float(dr[e]), __uint_as_float(dr[e + 1])));
           tmem_st8(tl + col_r(p ^ 1) + 8 * c, dd);
           // dS^T -> shared memory for dQ(t): block c/4, 16-byte chunks 2(c%4), 2(c%4)+1
           uint8_t* blk = dsrow + (c >> 2) * (BK * 128);

@@ -163,6 +163,13 @@ HD_DEVINLINE uint32_t cvt_bf16x2(float lo, float hi) {
   return r;
 }
 
+// Packed bf16 pair product, round to nearest even.
+HD_DEVINLINE uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("mul.rn.bf16x2 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
 // Packed fp32 pairs (Blackwell f32x2 ALU ops: one instruction, two lanes of math).
 HD_DEVINLINE uint64_t f2pack(float lo, float hi) {
   uint64_t r;
