@@ -25,10 +25,11 @@
 // TMEM: two 128-column regions R0, R1 swap roles with the tile parity p:
 //   S^T(t) in R[p] (P^T packed bf16 over its first 64 columns, then dQ(t)),
 //   dP^T(t) in R[p^1] (dS^T packed bf16 over its first 64 columns);  dV at 256, dK at 384.
-// MMA issue order:  for each quarter u of the query columns: wait P^T(t) quarter u |
-//                   dV(t) k-steps of u;  then per quarter: wait dS^T(t) quarter u | dK(t)
-//                   k-steps of u;  dQ(t) | wait R[p^1] pre-filled | S(t+1) | wait dQ(t)
-//                   read out and R[p] pre-filled | dP(t+1)
+// MMA issue order, issuer X:  for each quarter u of the query columns: wait P^T(t)
+//                   quarter u | dV(t) k-steps of u;  then per quarter: wait dS^T(t)
+//                   quarter u | dK(t) k-steps of u
+//                 issuer Y:  wait dS^T(t) complete and dV(t) done | dQ(t) | wait R[p^1]
+//                   pre-filled | S(t+1) | wait dQ(t) read out and R[p] pre-filled | dP(t+1)
 // Phase A of tile t+1 needs only S'^T(t+1), so it overlaps the dQ(t) read-out, the
 // dP(t+1) pre-fill and the dP(t+1) MMA; dV / dK k-steps run under the later quarters.
 // The pre-fills (every TMEM lane gets the same 128 per-query values) are written
@@ -38,12 +39,15 @@
 // one thread execute in order), so it overlaps the dQ(t) read-out; dP(t+1) lands in
 // R[p] only after that read-out.
 //
-// Roles (448 threads, at most 4 warps per scheduler so each thread keeps 128
-// registers): warp 0 TMA producer (+ TMEM owner), warp 1 MMA issuer, warps 2..5
-// softmax (TMEM lane = key row; 128 query columns in eight 16-column chunks),
-// warps 6..9 / 10..13 dQ flush and pre-fill for columns 0..63 / 64..127: each
-// loads its 64 dQ columns (TMEM lane = query row), pre-fills the region for the
-// next dP^T, then stages two 4 KB rounds through its own buffer.
+// Roles (480 threads, 128 registers each): warp 0 TMA producer (+ TMEM owner);
+// warp 1 MMA issuer X (dV, dK per query quarter); warp 14 MMA issuer Y (dQ, S, dP):
+// two issuing threads on different schedulers, because an MMA thread sharing its
+// scheduler with a busy softmax warp gets few issue slots, and one thread for all 40
+// MMAs and 12 barrier waits of a tile became the critical path; warps 2..5 softmax
+// (TMEM lane = key row; 128 query columns in eight 16-column chunks per phase);
+// warps 6..9 / 10..13 dQ flush and pre-fill for columns 0..63 / 64..127: each loads
+// its 64 dQ columns (TMEM lane = query row), pre-fills the region for the next dP^T,
+// then stages two 4 KB rounds through its own buffer.
 // Every mbarrier wait is bounded.
 #include "tc_common.cuh"
 
@@ -52,7 +56,7 @@ namespace hdsfa {
 typedef __nv_bfloat16 bf16;
 
 namespace tcbwd {
-constexpr int BK = 128, BQ = 128, DH = 128, NTHREADS = 448;
+constexpr int BK = 128, BQ = 128, DH = 128, NTHREADS = 480;
 constexpr uint32_t COL_DV = 256, COL_DK = 384;
 HD_DEVINLINE uint32_t col_r(int r) { return 128u * r; }
 
@@ -66,7 +70,7 @@ struct Smem {
   float nlse2[2][BQ];     // -lse*log2(e) of the query tile in q[i], loaded with it
   float ndelta[2][BQ];    // -delta of the query tile in q[i], loaded with it
   uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, pa_part[4], pb_part[4], dq_full, s_init,
-      dp_init, dk_done, kv_done, drain;
+      dp_init, dk_done, dv_done, kv_done, drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -127,7 +131,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       mbar_init(&sm.q_empty[i], 1);
     }
     mbar_init(&sm.do_full, 1);
-    mbar_init(&sm.do_empty, 1);
+    mbar_init(&sm.do_empty, 2);  // dV(t) (issuer X) and dP(t) (issuer Y) both read dO(t)
     mbar_init(&sm.s_full, 1);
     mbar_init(&sm.dp_full, 1);
     for (int i = 0; i < 4; ++i) {
@@ -138,8 +142,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     mbar_init(&sm.s_init, 256);
     mbar_init(&sm.dp_init, 256);
     mbar_init(&sm.dk_done, 1);
+    mbar_init(&sm.dv_done, 1);
     mbar_init(&sm.kv_done, 1);
-    mbar_init(&sm.drain, 1);
+    mbar_init(&sm.drain, 2);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -189,8 +194,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       for (int t = max(0, nq_issued - 2); t < nq_issued; ++t) mbar_drain(&sm.q_full[t & 1], (t >> 1) & 1);
       if (ndo_issued > 0) mbar_drain(&sm.do_full, (ndo_issued - 1) & 1);
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 || warp == NTHREADS / 32 - 1) {
+    // ------------------------------------------------------------ MMA issuers
     if (lane == 0) {
       constexpr uint32_t idSP = idesc_bf16(128, BQ, 0, 0);  // S^T, dP^T: A = K / V, B = Q / dO (K-major)
       constexpr uint32_t idKV = idesc_bf16(128, DH, 0, 1);  // dV, dK: A in TMEM, B = dO / Q MN-major
@@ -222,64 +227,84 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         for (int kk = k0; kk < k0 + 2; ++kk)
           tc_mma_ts(tmem + d_col, tmem + a_col + kk * 8, bd0 + moff(kk), idKV, (acc || kk > 0) ? 1u : 0u);
       };
-      bool ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.q_full[0], 0, abort, P.status) &&
-                mbar_wait(&sm.s_init, 0, abort, P.status);
-      if (ok) {
-        tc_fence_after();
-        issue_sp(kK, qK0, col_r(0));
-        tc_commit(&sm.s_full);
-        ok = mbar_wait(&sm.do_full, 0, abort, P.status) && mbar_wait(&sm.dp_init, 0, abort, P.status);
+      bool ok = true;
+      if (warp == 1) {
+        // ---- issuer X: dV(t) and dK(t), one query quarter at a time
+        for (int t = 0; ok && t < T; ++t) {
+          const int p = t & 1;
+          const uint64_t qM = p ? qM1 : qM0;
+          for (int u = 0; u < 4; ++u) {
+            if (!mbar_wait(&sm.pa_part[u], t & 1, abort, P.status)) { ok = false; break; }
+            tc_fence_after();
+            issue_kv(col_r(p), doM, COL_DV, t > 0, 2 * u);       // reads P^T(t) and dO(t)
+          }
+          if (!ok) break;
+          tc_commit(&sm.do_empty);
+          tc_commit(&sm.dv_done);  // issuer Y may write dQ(t) over P^T(t) in R[p]
+          for (int u = 0; u < 4; ++u) {
+            if (!mbar_wait(&sm.pb_part[u], t & 1, abort, P.status)) { ok = false; break; }
+            tc_fence_after();
+            issue_kv(col_r(p ^ 1), qM, COL_DK, t > 0, 2 * u);    // reads dS^T(t) and Q(t)
+          }
+          if (!ok) break;
+          tc_commit(&sm.q_empty[p]);
+          tc_commit(&sm.dk_done);  // R[p^1] free for the S'^T(t+1) pre-fill
+        }
+        tc_commit(&sm.kv_done);
+      } else {
+        // ---- issuer Y: S(0), dP(0), then per tile dQ(t), S(t+1), dP(t+1)
+        ok = mbar_wait(&sm.kv_full, 0, abort, P.status) && mbar_wait(&sm.q_full[0], 0, abort, P.status) &&
+             mbar_wait(&sm.s_init, 0, abort, P.status);
         if (ok) {
           tc_fence_after();
-          issue_sp(vK, doK, col_r(1));
-          tc_commit(&sm.dp_full);
-        }
-      }
-      for (int t = 0; ok && t < T; ++t) {
-        const int p = t & 1;
-        const uint64_t qM = p ? qM1 : qM0;
-        for (int u = 0; u < 4; ++u) {
-          if (!mbar_wait(&sm.pa_part[u], t & 1, abort, P.status)) { ok = false; break; }
-          tc_fence_after();
-          issue_kv(col_r(p), doM, COL_DV, t > 0, 2 * u);       // reads P^T(t) and dO(t)
-        }
-        if (!ok) break;
-        tc_commit(&sm.do_empty);
-        for (int u = 0; u < 4; ++u) {
-          if (!mbar_wait(&sm.pb_part[u], t & 1, abort, P.status)) { ok = false; break; }
-          tc_fence_after();
-          issue_kv(col_r(p ^ 1), qM, COL_DK, t > 0, 2 * u);    // reads dS^T(t) and Q(t)
-        }
-        if (!ok) break;
-        tc_commit(&sm.q_empty[p]);
-        tc_commit(&sm.dk_done);  // R[p^1] free for the S'^T(t+1) pre-fill
-        // dQ(t) = dS K into R[p] (after dV(t) and phase B(t) read P^T there)
-#pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk)
-          tc_mma_ss(tmem + col_r(p), dsM + moff(kk), kM + moff(kk), idQ, kk > 0 ? 1u : 0u);
-        tc_commit(&sm.dq_full);
-        if (t + 1 < T) {
-          // S^T(t+1) into R[p^1]: dK(t) has read dS^T(t) from it
-          if (!mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status) ||
-              !mbar_wait(&sm.s_init, (t + 1) & 1, abort, P.status)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          issue_sp(kK, p ? qK0 : qK1, col_r(p ^ 1));
+          issue_sp(kK, qK0, col_r(0));
           tc_commit(&sm.s_full);
-          // dP^T(t+1) into R[p]: dQ(t) read out and R[p] pre-filled, dO(t+1) loaded
-          if (!mbar_wait(&sm.dp_init, (t + 1) & 1, abort, P.status) ||
-              !mbar_wait(&sm.do_full, (t + 1) & 1, abort, P.status)) {
+          ok = mbar_wait(&sm.do_full, 0, abort, P.status) && mbar_wait(&sm.dp_init, 0, abort, P.status);
+          if (ok) {
+            tc_fence_after();
+            issue_sp(vK, doK, col_r(1));
+            tc_commit(&sm.dp_full);
+            tc_commit(&sm.do_empty);  // with issuer X's arrival after dV(0)
+          }
+        }
+        for (int t = 0; ok && t < T; ++t) {
+          const int p = t & 1;
+          // dQ(t) = dS K into R[p]: dS^T(t) complete in smem, phase B(t) and dV(t)
+          // (issuer X) done reading P^T(t) there
+          if (!mbar_wait(&sm.pb_part[3], t & 1, abort, P.status) ||
+              !mbar_wait(&sm.dv_done, t & 1, abort, P.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          issue_sp(vK, doK, col_r(p));
-          tc_commit(&sm.dp_full);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            tc_mma_ss(tmem + col_r(p), dsM + moff(kk), kM + moff(kk), idQ, kk > 0 ? 1u : 0u);
+          tc_commit(&sm.dq_full);
+          if (t + 1 < T) {
+            // S^T(t+1) into R[p^1]: s_init follows dK(t) (issuer X) having read dS^T(t) there
+            if (!mbar_wait(&sm.q_full[p ^ 1], ((t + 1) >> 1) & 1, abort, P.status) ||
+                !mbar_wait(&sm.s_init, (t + 1) & 1, abort, P.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_sp(kK, p ? qK0 : qK1, col_r(p ^ 1));
+            tc_commit(&sm.s_full);
+            // dP^T(t+1) into R[p]: dQ(t) read out and R[p] pre-filled, dO(t+1) loaded
+            if (!mbar_wait(&sm.dp_init, (t + 1) & 1, abort, P.status) ||
+                !mbar_wait(&sm.do_full, (t + 1) & 1, abort, P.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_sp(vK, doK, col_r(p));
+            tc_commit(&sm.dp_full);
+            tc_commit(&sm.do_empty);  // with issuer X's arrival after dV(t+1)
+          }
         }
       }
-      tc_commit(&sm.kv_done);
+      // every MMA either issuer started completes before TMEM / smem are released
       tc_commit(&sm.drain);
       mbar_drain(&sm.drain, 0);
     }
