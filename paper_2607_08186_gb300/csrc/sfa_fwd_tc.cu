@@ -241,18 +241,23 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
       const bool rescale = (m_run == -INFINITY) || ((m_new - m_run) * c2 > kRescaleThreshold);
       const float m_use = rescale ? m_new : m_run;
       const float neg = (m_use == -INFINITY) ? 0.f : -m_use * c2;
-      float sum[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) sum[e] = 0.f;
+      const uint64_t c2x2 = f2pack(c2, c2), neg2 = f2pack(neg, neg);
+      uint64_t sum2[4] = {0, 0, 0, 0};
       uint32_t pk[BN / 2];
 #pragma unroll
       for (int e = 0; e < BN; e += 2) {
-        const float p0 = ex2_approx(fmaf(x[e], c2, neg));
-        const float p1 = ex2_approx(fmaf(x[e + 1], c2, neg));
-        sum[(e >> 1) & 7] += p0 + p1;
+        float a0, a1;
+        f2unpack(ffma2(f2pack(x[e], x[e + 1]), c2x2, neg2), a0, a1);
+        const float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
+        sum2[(e >> 1) & 3] = fadd2(sum2[(e >> 1) & 3], f2pack(p0, p1));
         pk[e >> 1] = cvt_bf16x2(p0, p1);
       }
-      const float rsum = ((sum[0] + sum[1]) + (sum[2] + sum[3])) + ((sum[4] + sum[5]) + (sum[6] + sum[7]));
+      float s0, s1, s2, s3, s4, s5, s6, s7;
+      f2unpack(sum2[0], s0, s1);
+      f2unpack(sum2[1], s2, s3);
+      f2unpack(sum2[2], s4, s5);
+      f2unpack(sum2[3], s6, s7);
+      const float rsum = ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
       // O_g already holds every earlier tile's PV (its S of this tile was issued after them)
       const bool mine = rescale && m_run != -INFINITY && i > 0;
       if (__any_sync(0xffffffffu, mine)) {
