@@ -189,32 +189,71 @@ class HotPath:
                          for t in (self.o, self.lse, self.dq, self.dk, self.dv)]
         self.launches_per_step = 4 + (1 if with_gather else 0)
 
-    def step(self, ev=None):
+    def _bufs(self):
+        return {"q": self.q, "k": self.k, "v": self.v, "do": self.do, "ids": getattr(self, "ids", None),
+                "o": self.o, "lse": self.lse, "dq": self.dq, "dk": self.dk, "dv": self.dv}
+
+    def step(self, ev=None, bufs=None, stream=None):
         b, s = self.b, self.s
+        t = bufs or self._bufs()
         if self.with_gather:
-            b.hd_expand_embed(self.tables, self.ids, self.x)
+            b.hd_expand_embed(self.tables, t["ids"], self.x, stream=stream)
         if ev is not None:
             ev[0].record()
-        b.sfa_fwd(self.q, self.k, self.v, self.o, self.lse, s.n, self.mode)
+        b.sfa_fwd(t["q"], t["k"], t["v"], t["o"], t["lse"], s.n, self.mode, stream=stream)
         if ev is not None:
             ev[1].record()
-        b.sfa_bwd_prep(self.o, self.do, self.lse, s.n, self.mode, self.ws, s.Hkv)
+        b.sfa_bwd_prep(t["o"], t["do"], t["lse"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
         if ev is not None:
             ev[2].record()
-        b.sfa_bwd_main(self.q, self.k, self.v, self.do, self.dk, self.dv, s.n, self.mode, self.ws)
+        b.sfa_bwd_main(t["q"], t["k"], t["v"], t["do"], t["dk"], t["dv"], s.n, self.mode, self.ws,
+                       stream=stream)
         if ev is not None:
             ev[3].record()
-        b.sfa_bwd_finalize(self.dq, s.n, self.mode, self.ws, s.Hkv)
+        b.sfa_bwd_finalize(t["dq"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
 
-    def step_e2e(self):
-        """Host -> device inputs, the step, device -> host results (pinned buffers)."""
-        for dst, src in zip((self.q, self.k, self.v, self.do), self.host_in):
-            dst.copy_(src, non_blocking=True)
-        if self.with_gather:
-            self.ids.copy_(self.host_ids, non_blocking=True)
-        self.step()
-        for dst, src in zip(self.host_out, (self.o, self.lse, self.dq, self.dk, self.dv)):
-            dst.copy_(src, non_blocking=True)
+    def e2e(self, steps: int, warmup: int, ws: int) -> float:
+        """Seconds per step end to end with host buffers: every step copies its inputs
+        host -> device (pinned), runs the five launches and copies its results device ->
+        host.  Three streams overlap step k+1's upload and step k-1's download with step
+        k's compute; two device buffer sets, ordered by events, keep them apart."""
+        sets = [self._bufs()]
+        sets.append({name: (None if t is None else torch.empty_like(t)) for name, t in sets[0].items()})
+        s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+        n = warmup + steps
+        ev = {key: [torch.cuda.Event() for _ in range(n)] for key in ("in", "cmp", "out")}
+        ins = ("q", "k", "v", "do") + (("ids",) if self.with_gather else ())
+        host_in = list(self.host_in) + ([self.host_ids] if self.with_gather else [])
+        outs = ("o", "lse", "dq", "dk", "dv")
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        barrier(ws)
+        torch.cuda.synchronize()
+        for i in range(n):
+            if i == warmup:
+                s_in.wait_event(ev["out"][i - 1]) if i > 0 else None
+                t0.record(s_in)
+            d = sets[i & 1]
+            with torch.cuda.stream(s_in):
+                if i >= 2:
+                    s_in.wait_event(ev["cmp"][i - 2])  # step i-2 has read this set's inputs
+                for name, src in zip(ins, host_in):
+                    d[name].copy_(src, non_blocking=True)
+                ev["in"][i].record(s_in)
+            s_cmp.wait_event(ev["in"][i])
+            if i >= 2:
+                s_cmp.wait_event(ev["out"][i - 2])  # this set's previous results are out
+            self.step(bufs=d, stream=s_cmp)
+            ev["cmp"][i].record(s_cmp)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev["cmp"][i])
+                for dst, name in zip(self.host_out, outs):
+                    dst.copy_(d[name], non_blocking=True)
+                ev["out"][i].record(s_out)
+        t1.record(s_out)
+        torch.cuda.synchronize()
+        barrier(ws)
+        return t0.elapsed_time(t1) / 1e3 / steps
 
     def io_bytes(self):
         h2d = sum(t.numel() * t.element_size() for t in self.host_in)
@@ -433,7 +472,7 @@ def main():
     tr = traffic_record(dom)
 
     # end to end through the C ABI with host buffers
-    e2e_s = time_loop(hp.step_e2e, max(3, args.steps // 2), 2, ws)
+    e2e_s = hp.e2e(max(5, args.steps // 2), 3, ws)
     e2e_val, _ = job_throughput(flops_step, e2e_s, ws)
     h2d, d2h = hp.io_bytes()
     launches = hp.launches_per_step * args.steps
