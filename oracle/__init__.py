@@ -68,6 +68,12 @@ def _load():
             lib.hdo_stream_index.argtypes = [I64, I64]
             lib.hdo_expand.restype = I64
             lib.hdo_expand.argtypes = [P, P, P, I64, I64, I64, I64, I64]
+            lib.hdo_expand_bwd.restype = None
+            lib.hdo_expand_bwd.argtypes = [P, P, P, I64, I64, I64, I64, I64]
+            lib.hdo_select_final.restype = None
+            lib.hdo_select_final.argtypes = [P, P, I64, I64, I64, I64]
+            lib.hdo_select_final_bwd.restype = None
+            lib.hdo_select_final_bwd.argtypes = [P, P, I64, I64, I64, I64]
             D = ctypes.POINTER(_Dims)
             lib.hdo_sfa_fwd.argtypes = [P, P, P, P, P, D]
             lib.hdo_sfa_fwd_rows.argtypes = [P, P, P, D, I64, P, P, P]
@@ -131,6 +137,39 @@ def expand(tables: torch.Tensor, ids: torch.Tensor):
     out = np.empty((B, n * L, D), dtype=np.uint16)
     bad = _load().hdo_expand(_ptr(tb), _ptr(ib), _ptr(out), B, L, n, V, D)
     return torch.from_numpy(out.view(np.int16)).view(torch.bfloat16), int(bad)
+
+
+def expand_bwd(dX: torch.Tensor, ids: torch.Tensor, n: int, V: int, dE: torch.Tensor | None = None):
+    """Adjoint of the Eq. 1 gather: dE[k][x] += sum over tokens with id x of dX at
+    stream k.  dX [B][n*L][D] (any float dtype, upcast to fp64), ids [B][L] int32.
+    Returns dE fp64 [n][V][D] (a copy of `dE` plus the sums, or the sums alone)."""
+    B, nL, D = dX.shape
+    L = nL // n
+    xd = _f64(dX)
+    ib = np.ascontiguousarray(ids.detach().cpu().to(torch.int32).numpy())
+    out = np.zeros((n, V, D), dtype=np.float64) if dE is None else _f64(dE).copy()
+    _load().hdo_expand_bwd(_ptr(xd), _ptr(ib), _ptr(out), B, L, n, V, D)
+    return torch.from_numpy(out)
+
+
+def select_final(X: torch.Tensor, n: int):
+    """Eq. 2 final-stream rows: Y[b][i] = X[b][i*n + n-1] (bf16 bit copy)."""
+    B, nL, D = X.shape
+    L = nL // n
+    xb = np.ascontiguousarray(X.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16))
+    out = np.empty((B, L, D), dtype=np.uint16)
+    _load().hdo_select_final(_ptr(xb), _ptr(out), B, L, n, D)
+    return torch.from_numpy(out.view(np.int16)).view(torch.bfloat16)
+
+
+def select_final_bwd(dY: torch.Tensor, n: int):
+    """Adjoint of select_final: dY [B][L][D] bf16 back to the final-stream rows of a
+    zero [B][n*L][D] tensor."""
+    B, L, D = dY.shape
+    yb = np.ascontiguousarray(dY.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16))
+    out = np.empty((B, n * L, D), dtype=np.uint16)
+    _load().hdo_select_final_bwd(_ptr(yb), _ptr(out), B, L, n, D)
+    return torch.from_numpy(out.view(np.int16)).view(torch.bfloat16)
 
 
 def sfa_fwd(q, k, v, n: int, mode: int, scale: float | None = None, window: int = 0):

@@ -9,7 +9,10 @@
  * header, table or helper with the CUDA sources.
  *
  * What it computes (all citations are to the Hidden Decoding paper):
- *   - Eq. 1  : the expanded sequence S_t = E_k(x_i) at position t = (i-1)n + k.
+ *   - Eq. 1  : the expanded sequence S_t = E_k(x_i) at position t = (i-1)n + k, and
+ *              its adjoint (the gradient with respect to the n tables).
+ *   - Eq. 2  : the final-stream positions t = i n that the loss reads, and their
+ *              adjoint.
  *   - Eq. 3  : token index i(t) = ceil(t/n) and stream index s(t) = ((t-1) mod n) + 1.
  *   - Eq. 4  : the intra-stream mask M[t,t'] = 1[t' <= t and s(t') = s(t)] (WITHIN).
  *   - Fig. 2a: the full cross-stream layer, the standard causal mask over all
@@ -89,6 +92,47 @@ int64_t hdo_expand(const uint16_t* tables, const int32_t* ids, uint16_t* out,
     }
   }
   return bad;
+}
+
+/* ---- Eq. 1 backward: the adjoint of the expansion gather ----
+ * The forward copies E_k(x_i) to position t = (i-1)n + k, so the gradient of the
+ * loss with respect to row x of table k is the sum of the position gradients of
+ * every token i with x_i = x, taken at stream k:
+ *   dE_k[x] += sum_{i : x_i = x} dS_{(i-1)n+k}.
+ * dX: [B][n*L][D] fp64; ids: [B][L]; dE: [n][V][D] fp64, accumulated (not cleared).
+ * An id outside [0, V) contributes nothing (its rows were zero in the forward). */
+void hdo_expand_bwd(const double* dX, const int32_t* ids, double* dE, int64_t B, int64_t L,
+                    int64_t n, int64_t V, int64_t D) {
+  for (int64_t b = 0; b < B; ++b) {
+    for (int64_t i = 1; i <= L; ++i) {
+      int32_t x = ids[b * L + (i - 1)];
+      if (x < 0 || x >= V) continue;
+      for (int64_t k = 1; k <= n; ++k) {
+        int64_t t = (i - 1) * n + k;
+        const double* src = dX + (b * n * L + (t - 1)) * D;
+        double* dst = dE + ((k - 1) * V + x) * D;
+        for (int64_t c = 0; c < D; ++c) dst[c] += src[c];
+      }
+    }
+  }
+}
+
+/* ---- Eq. 2: the supervised (final-stream) positions ----
+ * Only the final stream of each token is supervised: the loss reads the hidden
+ * state at 1-indexed position t = i n.  select: Y[b][i-1] = X[b][i n - 1] (0-indexed
+ * rows of D bf16 bit patterns); its adjoint writes dY back to those rows and zero
+ * to every other position. */
+void hdo_select_final(const uint16_t* X, uint16_t* Y, int64_t B, int64_t L, int64_t n, int64_t D) {
+  for (int64_t b = 0; b < B; ++b)
+    for (int64_t i = 1; i <= L; ++i)
+      memcpy(Y + (b * L + (i - 1)) * D, X + (b * n * L + (i * n - 1)) * D, (size_t)D * sizeof(uint16_t));
+}
+
+void hdo_select_final_bwd(const uint16_t* dY, uint16_t* dX, int64_t B, int64_t L, int64_t n, int64_t D) {
+  memset(dX, 0, (size_t)(B * n * L * D) * sizeof(uint16_t));
+  for (int64_t b = 0; b < B; ++b)
+    for (int64_t i = 1; i <= L; ++i)
+      memcpy(dX + (b * n * L + (i * n - 1)) * D, dY + (b * L + (i - 1)) * D, (size_t)D * sizeof(uint16_t));
 }
 
 /* ---------------------------------------------------------------- helpers */

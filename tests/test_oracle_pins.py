@@ -6,6 +6,8 @@
 - Library routines: torch's fp64 scaled_dot_product_attention (forward) and its
   autograd (backward) for the special cases that reduce to textbook causal attention.
 - Exact special rows, probability-row invariants, and central finite differences.
+- Adjoint identities <A x, y> = <x, A^T y> for the Eq. 1 gather and the Eq. 2 final-stream
+  selection against their backward functions, plus torch index_add_ / indexing.
 """
 import math
 import os
@@ -131,6 +133,87 @@ def _brute_visible(t, tk, n, mode, w):
         return j < i or (j == i and r <= s)
     # Fig. 2b: causal window of w positions ending at the query (inclusive)
     return tk <= t and t - tk < w
+
+
+# ------------------------------------------------------------------ Eq. 1 backward, Eq. 2
+def _bf16_rand(shape, seed, scale=1.0):
+    return (_rand(shape, seed) * scale).to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("n", [1, 2, 4])
+def test_expand_bwd_is_adjoint_of_gather(n):
+    # <gather(E), dX> = <E, gather^T(dX)>: a wrong stream, token or row index breaks it
+    B, L, V, D = 2, 9, 13, 6
+    E = _bf16_rand((n, V, D), 300 + n)
+    g = torch.Generator().manual_seed(310 + n)
+    ids = torch.randint(0, V, (B, L), generator=g, dtype=torch.int32)
+    dX = _bf16_rand((B, n * L, D), 320 + n)
+    X, bad = oracle.expand(E, ids)
+    assert bad == 0
+    lhs = float((X.double() * dX.double()).sum())
+    rhs = float((E.double() * oracle.expand_bwd(dX, ids, n, V)).sum())
+    assert abs(lhs - rhs) <= 1e-12 * max(1.0, abs(lhs))
+
+
+def test_expand_bwd_matches_index_add():
+    B, L, n, V, D = 3, 17, 4, 11, 5
+    g = torch.Generator().manual_seed(330)
+    ids = torch.randint(0, V, (B, L), generator=g, dtype=torch.int32)
+    dX = _bf16_rand((B, n * L, D), 331)
+    ref = torch.zeros(n, V, D, dtype=torch.float64)
+    per_stream = dX.double().view(B, L, n, D)
+    for s in range(n):
+        ref[s].index_add_(0, ids.reshape(-1).long(), per_stream[:, :, s].reshape(-1, D))
+    assert torch.equal(oracle.expand_bwd(dX, ids, n, V), ref)
+
+
+def test_expand_bwd_repeated_id_and_accumulation():
+    # every token the same id: that row receives the sum over all tokens of its stream;
+    # an existing dE is added to, not replaced; other rows keep their values
+    B, L, n, V, D = 2, 7, 3, 5, 4
+    ids = torch.full((B, L), 2, dtype=torch.int32)
+    dX = _bf16_rand((B, n * L, D), 340)
+    dE0 = _rand((n, V, D), 341)
+    got = oracle.expand_bwd(dX, ids, n, V, dE=dE0)
+    want = dE0.clone()
+    want[:, 2] += dX.double().view(B, L, n, D).sum(dim=(0, 1))
+    assert torch.allclose(got, want, rtol=0, atol=1e-12)
+
+
+def test_expand_bwd_out_of_range_ids_contribute_nothing():
+    B, L, n, V, D = 1, 6, 2, 4, 3
+    ids = torch.tensor([[0, -1, 3, 4, 1, 1000]], dtype=torch.int32)
+    dX = _bf16_rand((B, n * L, D), 350)
+    got = oracle.expand_bwd(dX, ids, n, V)
+    keep = torch.tensor([0, 2, 4])  # tokens whose id is in range
+    ref = oracle.expand_bwd(dX.view(B, L, n, D)[:, keep].reshape(B, -1, D), ids[:, keep], n, V)
+    assert torch.equal(got, ref)
+
+
+@pytest.mark.parametrize("n", [1, 2, 4])
+def test_select_final_is_last_stream_rows(n):
+    # Eq. 2: the loss reads 1-indexed positions t = i n, i.e. stream n of every token
+    B, L, D = 2, 5, 6
+    X = _bf16_rand((B, n * L, D), 360 + n)
+    Y = oracle.select_final(X, n)
+    assert torch.equal(Y.view(torch.int16), X.view(B, L, n, D)[:, :, n - 1].contiguous().view(torch.int16))
+    rows = [i * n - 1 for i in range(1, L + 1)]  # 0-indexed positions t - 1 = i n - 1
+    assert torch.equal(Y.view(torch.int16), X[:, rows].contiguous().view(torch.int16))
+
+
+@pytest.mark.parametrize("n", [1, 3])
+def test_select_final_bwd_is_adjoint(n):
+    B, L, D = 2, 4, 5
+    X = _bf16_rand((B, n * L, D), 370 + n)
+    dY = _bf16_rand((B, L, D), 375 + n)
+    dX = oracle.select_final_bwd(dY, n)
+    lhs = float((oracle.select_final(X, n).double() * dY.double()).sum())
+    rhs = float((X.double() * dX.double()).sum())
+    assert abs(lhs - rhs) <= 1e-12 * max(1.0, abs(lhs))
+    # every position that is not a final stream receives zero
+    mask = torch.ones(B, L, n, dtype=torch.bool)
+    mask[:, :, n - 1] = False
+    assert not dX.view(B, L, n, D)[mask].any()
 
 
 @pytest.mark.parametrize("n", range(1, 9))
