@@ -122,19 +122,6 @@ def test_expand_out_of_range_zero_rows():
     assert torch.all(out[0, 6:8].float() == 0) and torch.all(out[0, 14:16].float() == 0)
 
 
-# ------------------------------------------------------------------ masks
-def _brute_visible(t, tk, n, mode, w):
-    """Independent characterisation on (token, stream) pairs, 1-indexed."""
-    i, s = (t - 1) // n + 1, (t - 1) % n + 1
-    j, r = (tk - 1) // n + 1, (tk - 1) % n + 1
-    if mode == oracle.WITHIN:   # Fig. 2c: streams invisible to each other, causal within a stream
-        return r == s and j <= i
-    if mode == oracle.CROSS:    # Fig. 2a: lower-triangular over positions = earlier token, or same token & earlier-or-same stream
-        return j < i or (j == i and r <= s)
-    # Fig. 2b: causal window of w positions ending at the query (inclusive)
-    return tk <= t and t - tk < w
-
-
 # ------------------------------------------------------------------ Eq. 1 backward, Eq. 2
 def _bf16_rand(shape, seed, scale=1.0):
     return (_rand(shape, seed) * scale).to(torch.bfloat16)
@@ -214,6 +201,19 @@ def test_select_final_bwd_is_adjoint(n):
     mask = torch.ones(B, L, n, dtype=torch.bool)
     mask[:, :, n - 1] = False
     assert not dX.view(B, L, n, D)[mask].any()
+
+
+# ------------------------------------------------------------------ masks
+def _brute_visible(t, tk, n, mode, w):
+    """Independent characterisation on (token, stream) pairs, 1-indexed."""
+    i, s = (t - 1) // n + 1, (t - 1) % n + 1
+    j, r = (tk - 1) // n + 1, (tk - 1) % n + 1
+    if mode == oracle.WITHIN:   # Fig. 2c: streams invisible to each other, causal within a stream
+        return r == s and j <= i
+    if mode == oracle.CROSS:    # Fig. 2a: lower-triangular over positions = earlier token, or same token & earlier-or-same stream
+        return j < i or (j == i and r <= s)
+    # Fig. 2b: causal window of w positions ending at the query (inclusive)
+    return tk <= t and t - tk < w
 
 
 @pytest.mark.parametrize("n", range(1, 9))
