@@ -45,7 +45,8 @@ typedef enum {
 } hd_status_t;
 
 /* Bits the kernels OR into *dev_status. */
-#define HD_DEVBIT_INDEX 1   /* a token id outside [0, V): its n output rows were zeroed */
+#define HD_DEVBIT_INDEX 1   /* a token id outside [0, V): hd_expand_embed zeroed its n output
+                               rows; hd_expand_embed_bwd left it out of the sums */
 #define HD_DEVBIT_TIMEOUT 2 /* a bounded pipeline wait expired; outputs are invalid */
 
 /* Attention mask of one SFA layer (Sec. 2.2, Eq. 4 and Fig. 2). */
@@ -65,6 +66,40 @@ typedef enum {
  */
 hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L, int n,
                             int V, int D, int32_t* dev_status, cudaStream_t stream);
+
+/*
+ * hd_expand_embed_bwd -- backward of the expansion (adjoint of Eq. 1, Sec. 2.1):
+ *   dtables[s][v][:] += sum over (b, t) with ids[b][t] = v of dout[b][t*n + s][:]
+ * for every s < n and every v in [0, V) that occurs in ids.
+ *   dout: bf16 [B][n*L][D] (read-only); ids: int32 [B][L]; dtables: float32 [n][V][D],
+ *   accumulated in place (rows of ids that do not occur are not touched; zero the
+ *   tables first for a plain gradient).
+ *   Deterministic: every element of dtables is written by one thread, which adds the
+ *   occurrences of its id in ascending token order (b*L + t) in fp32 and then adds
+ *   that sum to dtables: repeated calls on the same inputs give identical bits.
+ *   An id outside [0, V) contributes nothing and sets HD_DEVBIT_INDEX.
+ *   workspace: device memory of at least hd_expand_embed_bwd_workspace_bytes(B, L)
+ *   bytes, 16-byte aligned, overwritten (no contents need to survive between calls).
+ *   Requires D % 8 == 0, B*L < 2^31, n*D < 2^31, 16-byte aligned dout/dtables;
+ *   HBM-bound.
+ */
+size_t hd_expand_embed_bwd_workspace_bytes(int B, int L); /* 0 for invalid sizes */
+hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dtables, int B, int L,
+                                int n, int V, int D, void* workspace, size_t workspace_bytes,
+                                int32_t* dev_status, cudaStream_t stream);
+
+/*
+ * hd_select_final_stream -- the positions the loss reads (Eq. 2, Sec. 2.1): the loss
+ * is taken only on each token's final stream, 0-indexed position t*n + n-1.
+ *   y[b][t][:] = x[b][t*n + n-1][:]   x: bf16 [B][n*L][D], y: bf16 [B][L][D].
+ * hd_select_final_stream_bwd -- its adjoint:
+ *   dx[b][t*n + n-1][:] = dy[b][t][:], every other row of dx is set to zero.
+ * Bit-exact copies; D % 8 == 0, 16-byte aligned pointers; HBM-bound.
+ */
+hd_status_t hd_select_final_stream(const void* x, void* y, int B, int L, int n, int D,
+                                   cudaStream_t stream);
+hd_status_t hd_select_final_stream_bwd(const void* dy, void* dx, int B, int L, int n, int D,
+                                       cudaStream_t stream);
 
 /*
  * sfa_fwd -- SFA forward over the expanded sequence (Sec. 2.2; Eq. 3-4; Fig. 2):

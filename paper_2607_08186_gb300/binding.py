@@ -43,6 +43,14 @@ def lib():
             P, I, F, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
             L.hd_expand_embed.restype = I
             L.hd_expand_embed.argtypes = [P, P, P, I, I, I, I, I, P, P]
+            L.hd_expand_embed_bwd_workspace_bytes.restype = Z
+            L.hd_expand_embed_bwd_workspace_bytes.argtypes = [I, I]
+            L.hd_expand_embed_bwd.restype = I
+            L.hd_expand_embed_bwd.argtypes = [P, P, P, I, I, I, I, I, P, Z, P, P]
+            L.hd_select_final_stream.restype = I
+            L.hd_select_final_stream.argtypes = [P, P, I, I, I, I, P]
+            L.hd_select_final_stream_bwd.restype = I
+            L.hd_select_final_stream_bwd.argtypes = [P, P, I, I, I, I, P]
             L.sfa_fwd.restype = I
             L.sfa_fwd.argtypes = [P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, P]
             L.sfa_bwd_workspace_bytes.restype = Z
@@ -90,6 +98,44 @@ def hd_expand_embed(tables, ids, out, dev_status=None, stream=None):
     _check(lib().hd_expand_embed(_p(tables), _p(ids), _p(out), B, L, n, V, D, _p(dev_status),
                                  _stream(stream)), "hd_expand_embed")
     return out
+
+
+def hd_expand_embed_bwd_workspace_bytes(B, L) -> int:
+    return int(lib().hd_expand_embed_bwd_workspace_bytes(B, L))
+
+
+def hd_expand_embed_bwd(dout, ids, dtables, workspace, dev_status=None, stream=None):
+    """dtables[s][v] += sum of dout[b][t*n+s] over tokens with ids[b][t] = v (adjoint of Eq. 1).
+    dout [B][n*L][D] bf16, ids [B][L] int32, dtables [n][V][D] float32 (accumulated in place),
+    workspace: uint8 CUDA tensor of >= hd_expand_embed_bwd_workspace_bytes(B, L) bytes."""
+    n, V, D = dtables.shape
+    B, L = ids.shape
+    if dout.shape[1] != n * L:
+        raise ValueError("dout.shape[1] must be n * L")
+    _check(lib().hd_expand_embed_bwd(_p(dout), _p(ids), _p(dtables), B, L, n, V, D, _p(workspace),
+                                     _wsb(workspace), _p(dev_status), _stream(stream)),
+           "hd_expand_embed_bwd")
+    return dtables
+
+
+def hd_select_final_stream(x, y, n, stream=None):
+    """y[b][t] = x[b][t*n + n-1], the rows the loss reads (Eq. 2).  x [B][n*L][D], y [B][L][D] bf16."""
+    B, L, D = y.shape
+    if x.shape[1] != n * L:
+        raise ValueError("x.shape[1] must be n * L")
+    _check(lib().hd_select_final_stream(_p(x), _p(y), B, L, n, D, _stream(stream)),
+           "hd_select_final_stream")
+    return y
+
+
+def hd_select_final_stream_bwd(dy, dx, n, stream=None):
+    """dx[b][t*n + n-1] = dy[b][t], zero elsewhere.  dy [B][L][D], dx [B][n*L][D] bf16."""
+    B, L, D = dy.shape
+    if dx.shape[1] != n * L:
+        raise ValueError("dx.shape[1] must be n * L")
+    _check(lib().hd_select_final_stream_bwd(_p(dy), _p(dx), B, L, n, D, _stream(stream)),
+           "hd_select_final_stream_bwd")
+    return dx
 
 
 def _attn_dims(q, k, n):

@@ -9,6 +9,11 @@
 namespace hdsfa {
 cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L,
                                 int n, int V, int D, int32_t* status, cudaStream_t stream);
+long long expand_bwd_sort_len(long long N);
+cudaError_t launch_expand_bwd(const void* dx, const int32_t* ids, float* de, int B, int L, int n, int V, int D,
+                              void* keys_ws, int32_t* status, cudaStream_t st);
+cudaError_t launch_select_final(const void* x, void* y, int B, int L, int n, int D, cudaStream_t st);
+cudaError_t launch_select_final_bwd(const void* dy, void* dx, int B, int L, int n, int D, cudaStream_t st);
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
                               const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
@@ -118,6 +123,36 @@ hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, i
   return hdsfa::launch_expand_embed(tables, ids, out, B, L, n, V, D, dev_status, stream) == cudaSuccess
              ? HD_OK
              : HD_ERR_CUDA;
+}
+
+size_t hd_expand_embed_bwd_workspace_bytes(int B, int L) {
+  if (B <= 0 || L <= 0 || (long long)B * L >= (1LL << 31)) return 0;
+  return (size_t)hdsfa::expand_bwd_sort_len((long long)B * L) * sizeof(unsigned long long);
+}
+
+hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dtables, int B, int L, int n,
+                                int V, int D, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                                cudaStream_t stream) {
+  if (!aligned16(dout) || !aligned16(dtables) || ids == nullptr) return HD_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || n <= 0 || V <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
+  const size_t need = hd_expand_embed_bwd_workspace_bytes(B, L);
+  if (need == 0 || (long long)n * D >= (1LL << 31)) return HD_ERR_UNSUPPORTED;
+  if (!aligned16(workspace) || workspace_bytes < need) return HD_ERR_WORKSPACE;
+  return cuda_status(hdsfa::launch_expand_bwd(dout, ids, dtables, B, L, n, V, D, workspace, dev_status, stream));
+}
+
+hd_status_t hd_select_final_stream(const void* x, void* y, int B, int L, int n, int D, cudaStream_t stream) {
+  if (!aligned16(x) || !aligned16(y)) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || n <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
+  return cuda_status(hdsfa::launch_select_final(x, y, B, L, n, D, stream));
+}
+
+hd_status_t hd_select_final_stream_bwd(const void* dy, void* dx, int B, int L, int n, int D,
+                                       cudaStream_t stream) {
+  if (!aligned16(dy) || !aligned16(dx)) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || n <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
+  return cuda_status(hdsfa::launch_select_final_bwd(dy, dx, B, L, n, D, stream));
 }
 
 hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,

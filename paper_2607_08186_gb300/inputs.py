@@ -72,3 +72,21 @@ def embed_inputs(B: int, L: int, n: int, V: int, D: int, seed: int = 0):
     g.manual_seed(seed + 1000)
     ids = torch.randint(0, V, (B, L), generator=g, dtype=torch.int64).to(torch.int32)
     return tables, ids
+
+
+def normal_bf16(shape, seed: int, std: float = 1.0) -> torch.Tensor:
+    """bf16 tensor ~ N(0, std^2) from a seeded CPU generator (gradients of the expanded rows)."""
+    return _randn(tuple(shape), seed, std=std)
+
+
+def token_ids(B: int, L: int, V: int, seed: int, zipf: float = 0.0) -> torch.Tensor:
+    """Token ids int32 [B][L].  zipf = 0: U[0, V).  zipf = a > 0: P(id = r) proportional to
+    (r + 1)^-a, the rank-frequency shape of natural-language tokens, so frequent ids repeat
+    many times within a batch (ranks are taken as ids; no permutation)."""
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed + 2000)
+    if zipf <= 0.0:
+        return torch.randint(0, V, (B, L), generator=g, dtype=torch.int64).to(torch.int32)
+    w = torch.arange(1, V + 1, dtype=torch.float64).pow(-zipf)
+    ids = torch.multinomial(w, B * L, replacement=True, generator=g)
+    return ids.view(B, L).to(torch.int32)

@@ -91,3 +91,37 @@ def test_expand_validation(lib):
     assert lib.hd_expand_embed(P(FAKE), P(FAKE), P(FAKE + 2), 1, 4, 2, 16, 16, None, None) == 1
     assert lib.hd_expand_embed(P(FAKE), None, P(FAKE), 1, 4, 2, 16, 16, None, None) == 1
     assert lib.hd_expand_embed(P(FAKE), P(FAKE), P(FAKE), 1, 4, 0, 16, 16, None, None) == 1
+
+
+def test_expand_bwd_workspace_size(lib):
+    assert lib.hd_expand_embed_bwd_workspace_bytes(1, 1) == 2048 * 8      # one shared-memory block of keys
+    assert lib.hd_expand_embed_bwd_workspace_bytes(1, 4096) == 4096 * 8
+    assert lib.hd_expand_embed_bwd_workspace_bytes(3, 1500) == 8192 * 8   # next power of two
+    assert lib.hd_expand_embed_bwd_workspace_bytes(0, 4) == 0
+    assert lib.hd_expand_embed_bwd_workspace_bytes(1 << 16, 1 << 15) == 0  # B*L must stay below 2^31
+
+
+def test_expand_bwd_validation(lib):
+    P, Z = ctypes.c_void_p, ctypes.c_size_t
+    ws = lib.hd_expand_embed_bwd_workspace_bytes(1, 4)
+
+    def call(dout=FAKE, ids=FAKE, de=FAKE, B=1, L=4, n=2, V=16, D=16, w=FAKE, wb=ws):
+        return lib.hd_expand_embed_bwd(P(dout), P(ids), P(de), B, L, n, V, D, P(w), Z(wb), None, None)
+
+    assert call(D=12) == 1                     # D % 8
+    assert call(dout=FAKE + 2) == 1            # misaligned
+    assert call(ids=0) == 1                    # null ids
+    assert call(ids=FAKE + 2) == 1             # ids not 4-byte aligned
+    assert call(n=0) == 1 and call(V=0) == 1 and call(B=0) == 1
+    assert call(wb=ws - 8) == 4                # workspace too small
+    assert call(w=0) == 4
+    assert call(n=1 << 20, D=1 << 12) == 2     # n*D beyond 2^31
+
+
+def test_select_final_validation(lib):
+    P = ctypes.c_void_p
+    for f in (lib.hd_select_final_stream, lib.hd_select_final_stream_bwd):
+        assert f(P(FAKE), P(FAKE), 1, 4, 2, 12, None) == 1
+        assert f(P(FAKE + 4), P(FAKE), 1, 4, 2, 16, None) == 1
+        assert f(P(FAKE), None, 1, 4, 2, 16, None) == 1
+        assert f(P(FAKE), P(FAKE), 1, 0, 2, 16, None) == 1
