@@ -10,8 +10,10 @@ Metric: attention FLOPs over visible pairs only (forward 4*Dh, backward 10*Dh pe
 pair and query head) per second of the whole step, in TFLOP/s.
 
 The same JSON line also carries: the dominant kernel's roofline, the end-to-end
-number through the C ABI with host buffers, the CPU oracle baseline, the CROSS
-(full cross-stream) layer of the same shape and the expansion-factor sweep.
+number through the C ABI with host buffers, the CPU oracle baseline, and under
+"extras" the CROSS (full cross-stream) layer of the same shape, the expansion-factor
+sweep, the LOCAL (sliding-window) layer at windows of 1024 and 4096 positions, and
+the HBM bandwidth of the expansion backward and the final-stream selection.
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the paper publishes no implementation to run).
@@ -161,10 +163,10 @@ class ClockSampler:
 class HotPath:
     """Device buffers and the five launches of one step."""
 
-    def __init__(self, s: AttnShape, mode: int, dev, with_gather: bool = True, seed: int = 1):
+    def __init__(self, s: AttnShape, mode: int, dev, with_gather: bool = True, seed: int = 1, window: int = 0):
         from paper_2607_08186_gb300 import binding
         self.b = binding
-        self.s, self.mode, self.dev = s, mode, dev
+        self.s, self.mode, self.dev, self.window = s, mode, dev, window
         q, k, v, do = attn_inputs(s, seed=seed)
         self.host_in = [t.pin_memory() for t in (q, k, v, do)]
         self.q, self.k, self.v, self.do = (t.to(dev, non_blocking=False) for t in self.host_in)
@@ -200,14 +202,14 @@ class HotPath:
             b.hd_expand_embed(self.tables, t["ids"], self.x, stream=stream)
         if ev is not None:
             ev[0].record()
-        b.sfa_fwd(t["q"], t["k"], t["v"], t["o"], t["lse"], s.n, self.mode, stream=stream)
+        b.sfa_fwd(t["q"], t["k"], t["v"], t["o"], t["lse"], s.n, self.mode, window=self.window, stream=stream)
         if ev is not None:
             ev[1].record()
         b.sfa_bwd_prep(t["o"], t["do"], t["lse"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
         if ev is not None:
             ev[2].record()
         b.sfa_bwd_main(t["q"], t["k"], t["v"], t["do"], t["dk"], t["dv"], s.n, self.mode, self.ws,
-                       stream=stream)
+                       window=self.window, stream=stream)
         if ev is not None:
             ev[3].record()
         b.sfa_bwd_finalize(t["dq"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
@@ -279,9 +281,9 @@ def time_loop(fn, steps, warmup, ws):
     return t0.elapsed_time(t1) / 1e3 / steps
 
 
-def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2):
+def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2, window: int = 0):
     """fwd, bwd-main and fwd+bwd times of one layer (no gather), seconds."""
-    hp = HotPath(s, mode, dev, with_gather=False, seed=7)
+    hp = HotPath(s, mode, dev, with_gather=False, seed=7, window=window)
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(iters)]
     for _ in range(warmup):
         hp.step()
@@ -298,6 +300,79 @@ def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2):
     del hp
     torch.cuda.empty_cache()
     return {"fwd_s": fwd, "bwd_main_s": bwd, "step_s": total}
+
+
+# ---------------------------------------------------------------- bandwidth ops
+_FLUSH = None
+
+
+def flush_l2(dev):
+    """Overwrite a 256 MB buffer (twice the 129 MB L2) so the next launch reads from HBM."""
+    global _FLUSH
+    if _FLUSH is None:
+        _FLUSH = torch.empty(64 << 20, dtype=torch.float32, device=dev)
+    _FLUSH.fill_(1.0)
+
+
+def time_op(fn, dev, iters=10, warmup=3):
+    """Median device time (s) of fn(), each call timed alone after an L2 flush."""
+    for _ in range(warmup):
+        fn()
+    ts = []
+    for _ in range(iters):
+        flush_l2(dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b) / 1e3)
+    return statistics.median(ts)
+
+
+def measure_expansion_backward(dev, hbm_peak: float):
+    """Expansion backward (adjoint of Eq. 1) and final-stream selection (Eq. 2) with
+    its adjoint at the step's shapes: L=4096 tokens, n=4, D=4096, V=151936.
+    Algorithmic bytes: expansion backward reads dX (n*L*D bf16) and the ids and
+    reads + writes the fp32 rows of the distinct ids (U*n*D*8); its apply part (the
+    row sums after the id-only plan) the same without the ids; selection reads and
+    writes L*D bf16; its adjoint reads L*D and writes n*L*D bf16."""
+    from paper_2607_08186_gb300 import binding, inputs
+    B, L, n, V, D = 1, 4096, 4, GATHER_V, GATHER_D
+    g = torch.Generator(device=dev)
+    g.manual_seed(31)
+    dX = torch.randn(B, n * L, D, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    dE = torch.zeros(n, V, D, dtype=torch.float32, device=dev)
+    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device=dev)
+    out = {}
+    for name, zipf in (("uniform_ids", 0.0), ("zipf1_ids", 1.0)):
+        ids = inputs.token_ids(B, L, V, seed=31, zipf=zipf).to(dev)
+        U = int(torch.unique(ids).numel())
+        t = time_op(lambda: binding.hd_expand_embed_bwd(dX, ids, dE, ws), dev)
+        nbytes = B * n * L * D * 2 + B * L * 4 + U * n * D * 8
+        binding.hd_expand_embed_bwd_plan(ids, V, ws)
+        t_apply = time_op(lambda: binding.hd_expand_embed_bwd_apply(dX, dE, ws, L), dev)
+        t_plan = time_op(lambda: binding.hd_expand_embed_bwd_plan(ids, V, ws), dev)
+        ab = nbytes - B * L * 4
+        out[f"expand_bwd_{name}"] = {"ms": t * 1e3, "distinct_ids": U, "bytes": nbytes,
+                                     "gbs": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / hbm_peak,
+                                     "plan_ms": t_plan * 1e3, "apply_ms": t_apply * 1e3,
+                                     "apply_gbs": ab / t_apply / 1e9,
+                                     "apply_frac_hbm": ab / t_apply / 1e9 / hbm_peak}
+    del dE
+    y = torch.empty(B, L, D, dtype=torch.bfloat16, device=dev)
+    t = time_op(lambda: binding.hd_select_final_stream(dX, y, n), dev)
+    nbytes = 2 * B * L * D * 2
+    out["select_final"] = {"ms": t * 1e3, "bytes": nbytes, "gbs": nbytes / t / 1e9,
+                           "frac_hbm": nbytes / t / 1e9 / hbm_peak}
+    t = time_op(lambda: binding.hd_select_final_stream_bwd(y, dX, n), dev)
+    nbytes = B * L * D * 2 + B * n * L * D * 2
+    out["select_final_bwd"] = {"ms": t * 1e3, "bytes": nbytes, "gbs": nbytes / t / 1e9,
+                               "frac_hbm": nbytes / t / 1e9 / hbm_peak}
+    out["workload"] = f"B={B} L={L} n={n} V={V} D={D}, inputs flushed from L2 before each launch"
+    del dX, y, ws
+    torch.cuda.empty_cache()
+    return out
 
 
 # ---------------------------------------------------------------- ncu traffic record
@@ -404,8 +479,8 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--no-extras", action="store_true", help="skip CROSS layer, n sweep and CPU baseline")
-    ap.add_argument("--layer-only", choices=["within", "cross"], default=None,
+    ap.add_argument("--no-extras", action="store_true", help="skip the extras (CROSS / LOCAL layers, n sweep, expansion backward) and the CPU baseline")
+    ap.add_argument("--layer-only", choices=["within", "cross", "local"], default=None,
                     help="time only one attention layer (fwd + bwd, no gather / e2e / extras); "
                          "the small case used for kernel profiles")
     args = ap.parse_args()
@@ -425,9 +500,10 @@ def main():
     s = SHAPES[WORKLOAD]
     pk = peaks()
     if args.layer_only:
-        mode = WITHIN if args.layer_only == "within" else CROSS
-        r = measure_layer(s, mode, dev, iters=args.steps, warmup=args.warmup)
-        fl = attn_flops(s, mode, FWD_FLOP + BWD_FLOP)
+        mode = {"within": WITHIN, "cross": CROSS, "local": LOCAL}[args.layer_only]
+        w = 4096 if mode == LOCAL else 0
+        r = measure_layer(s, mode, dev, iters=args.steps, warmup=args.warmup, window=w)
+        fl = attn_flops(s, mode, FWD_FLOP + BWD_FLOP, w)
         if rank == 0:
             print(json.dumps({"layer": f"{WORKLOAD}_{args.layer_only}", "ms": r["step_s"] * 1e3,
                               "tflops": fl / r["step_s"] / 1e12, "fwd_ms": r["fwd_s"] * 1e3,
@@ -522,6 +598,15 @@ def main():
         for row in sweep:
             row["WITHIN_cost_vs_n1"] = row["WITHIN"]["ms"] / base
         extras["n_sweep"] = sweep
+        loc = []
+        for w in (1024, 4096):
+            r = measure_layer(s, LOCAL, dev, window=w)
+            fl = attn_flops(s, LOCAL, FWD_FLOP + BWD_FLOP, w)
+            loc.append({"window_positions": w, "ms": r["step_s"] * 1e3, "tflops": fl / r["step_s"] / 1e12,
+                        "fwd_tflops": attn_flops(s, LOCAL, FWD_FLOP, w) / r["fwd_s"] / 1e12,
+                        "bwd_main_tflops": attn_flops(s, LOCAL, BWD_FLOP, w) / r["bwd_main_s"] / 1e12})
+        extras["local_layer"] = {"workload": f"{WORKLOAD}_local", "windows": loc}
+        extras["expansion_backward"] = measure_expansion_backward(dev, pk["hbm"])
         out["extras"] = extras
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:

@@ -74,12 +74,16 @@ hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, i
  *   dout: bf16 [B][n*L][D] (read-only); ids: int32 [B][L]; dtables: float32 [n][V][D],
  *   accumulated in place (rows of ids that do not occur are not touched; zero the
  *   tables first for a plain gradient).
- *   Deterministic: every element of dtables is written by one thread, which adds the
- *   occurrences of its id in ascending token order (b*L + t) in fp32 and then adds
- *   that sum to dtables: repeated calls on the same inputs give identical bits.
+ *   Deterministic: every element of dtables is read and written once, by one thread,
+ *   which sums the occurrences of its id in fp32 in an order fixed by their number
+ *   (ascending token order b*L + t; for ids with more than 32 occurrences, eight
+ *   consecutive token blocks, each in ascending order, whose sums are added in
+ *   block order) and adds the sum to dtables: repeated calls on the same inputs give
+ *   identical bits.
  *   An id outside [0, V) contributes nothing and sets HD_DEVBIT_INDEX.
  *   workspace: device memory of at least hd_expand_embed_bwd_workspace_bytes(B, L)
- *   bytes, 16-byte aligned, overwritten (no contents need to survive between calls).
+ *   bytes, 16-byte aligned, overwritten (no contents need to survive between calls;
+ *   the size is independent of n, V and D).
  *   Requires D % 8 == 0, B*L < 2^31, n*D < 2^31, 16-byte aligned dout/dtables;
  *   HBM-bound.
  */
@@ -87,6 +91,20 @@ size_t hd_expand_embed_bwd_workspace_bytes(int B, int L); /* 0 for invalid sizes
 hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dtables, int B, int L,
                                 int n, int V, int D, void* workspace, size_t workspace_bytes,
                                 int32_t* dev_status, cudaStream_t stream);
+/*
+ * The same in two parts.  hd_expand_embed_bwd_plan reads only ids: it sorts the
+ * tokens by id and lists each id's run of tokens in the workspace (the "plan"), so a
+ * caller can build it as soon as the ids are known (e.g. on a side stream during the
+ * forward pass) and keep it for several applies.  hd_expand_embed_bwd_apply adds the
+ * gradient rows into dtables following a plan of the same ids, B, L and V; the
+ * workspace must hold that plan, unmodified, when the apply runs (order a plan on
+ * another stream before the apply with an event).  plan + apply == hd_expand_embed_bwd.
+ */
+hd_status_t hd_expand_embed_bwd_plan(const int32_t* ids, int B, int L, int V, void* workspace,
+                                     size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream);
+hd_status_t hd_expand_embed_bwd_apply(const void* dout, float* dtables, int B, int L, int n, int V,
+                                      int D, const void* workspace, size_t workspace_bytes,
+                                      cudaStream_t stream);
 
 /*
  * hd_select_final_stream -- the positions the loss reads (Eq. 2, Sec. 2.1): the loss

@@ -47,6 +47,10 @@ def lib():
             L.hd_expand_embed_bwd_workspace_bytes.argtypes = [I, I]
             L.hd_expand_embed_bwd.restype = I
             L.hd_expand_embed_bwd.argtypes = [P, P, P, I, I, I, I, I, P, Z, P, P]
+            L.hd_expand_embed_bwd_plan.restype = I
+            L.hd_expand_embed_bwd_plan.argtypes = [P, I, I, I, P, Z, P, P]
+            L.hd_expand_embed_bwd_apply.restype = I
+            L.hd_expand_embed_bwd_apply.argtypes = [P, P, I, I, I, I, I, P, Z, P]
             L.hd_select_final_stream.restype = I
             L.hd_select_final_stream.argtypes = [P, P, I, I, I, I, P]
             L.hd_select_final_stream_bwd.restype = I
@@ -115,6 +119,26 @@ def hd_expand_embed_bwd(dout, ids, dtables, workspace, dev_status=None, stream=N
     _check(lib().hd_expand_embed_bwd(_p(dout), _p(ids), _p(dtables), B, L, n, V, D, _p(workspace),
                                      _wsb(workspace), _p(dev_status), _stream(stream)),
            "hd_expand_embed_bwd")
+    return dtables
+
+
+def hd_expand_embed_bwd_plan(ids, V, workspace, dev_status=None, stream=None):
+    """The id-only part of hd_expand_embed_bwd: tokens sorted by id and each id's run,
+    written into workspace for later hd_expand_embed_bwd_apply calls."""
+    B, L = ids.shape
+    _check(lib().hd_expand_embed_bwd_plan(_p(ids), B, L, int(V), _p(workspace), _wsb(workspace),
+                                          _p(dev_status), _stream(stream)), "hd_expand_embed_bwd_plan")
+
+
+def hd_expand_embed_bwd_apply(dout, dtables, workspace, L, stream=None):
+    """dtables += the expansion backward of dout following the plan held in workspace
+    (built by hd_expand_embed_bwd_plan for the same ids, B = dout.shape[0], L and V)."""
+    n, V, D = dtables.shape
+    B = dout.shape[0]
+    if dout.shape[1] != n * L:
+        raise ValueError("dout.shape[1] must be n * L")
+    _check(lib().hd_expand_embed_bwd_apply(_p(dout), _p(dtables), B, L, n, V, D, _p(workspace),
+                                           _wsb(workspace), _stream(stream)), "hd_expand_embed_bwd_apply")
     return dtables
 
 

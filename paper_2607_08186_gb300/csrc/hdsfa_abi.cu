@@ -9,9 +9,11 @@
 namespace hdsfa {
 cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L,
                                 int n, int V, int D, int32_t* status, cudaStream_t stream);
-long long expand_bwd_sort_len(long long N);
-cudaError_t launch_expand_bwd(const void* dx, const int32_t* ids, float* de, int B, int L, int n, int V, int D,
-                              void* keys_ws, int32_t* status, cudaStream_t st);
+size_t expand_bwd_ws_bytes(long long N);
+cudaError_t launch_expand_bwd_plan(const int32_t* ids, int B, int L, int V, void* ws, int32_t* status,
+                                   cudaStream_t st);
+cudaError_t launch_expand_bwd_apply(const void* dx, float* de, int B, int L, int n, int V, int D, const void* ws,
+                                    cudaStream_t st);
 cudaError_t launch_select_final(const void* x, void* y, int B, int L, int n, int D, cudaStream_t st);
 cudaError_t launch_select_final_bwd(const void* dy, void* dx, int B, int L, int n, int D, cudaStream_t st);
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
@@ -127,19 +129,42 @@ hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, i
 
 size_t hd_expand_embed_bwd_workspace_bytes(int B, int L) {
   if (B <= 0 || L <= 0 || (long long)B * L >= (1LL << 31)) return 0;
-  return (size_t)hdsfa::expand_bwd_sort_len((long long)B * L) * sizeof(unsigned long long);
+  return hdsfa::expand_bwd_ws_bytes((long long)B * L);
+}
+
+hd_status_t hd_expand_embed_bwd_plan(const int32_t* ids, int B, int L, int V, void* workspace,
+                                     size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream) {
+  if (ids == nullptr || (reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || V <= 0) return HD_ERR_INVALID_ARG;
+  const size_t need = hd_expand_embed_bwd_workspace_bytes(B, L);
+  if (need == 0) return HD_ERR_UNSUPPORTED;
+  if (!aligned16(workspace) || workspace_bytes < need) return HD_ERR_WORKSPACE;
+  return cuda_status(hdsfa::launch_expand_bwd_plan(ids, B, L, V, workspace, dev_status, stream));
+}
+
+hd_status_t hd_expand_embed_bwd_apply(const void* dout, float* dtables, int B, int L, int n, int V, int D,
+                                      const void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  if (!aligned16(dout) || !aligned16(dtables)) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || n <= 0 || V <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
+  const size_t need = hd_expand_embed_bwd_workspace_bytes(B, L);
+  if (need == 0 || (long long)n * D >= (1LL << 31)) return HD_ERR_UNSUPPORTED;
+  if (!aligned16(workspace) || workspace_bytes < need) return HD_ERR_WORKSPACE;
+  return cuda_status(hdsfa::launch_expand_bwd_apply(dout, dtables, B, L, n, V, D, workspace, stream));
 }
 
 hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dtables, int B, int L, int n,
                                 int V, int D, void* workspace, size_t workspace_bytes, int32_t* dev_status,
                                 cudaStream_t stream) {
+  // every argument is checked before the plan is enqueued
   if (!aligned16(dout) || !aligned16(dtables) || ids == nullptr) return HD_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || n <= 0 || V <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
   const size_t need = hd_expand_embed_bwd_workspace_bytes(B, L);
   if (need == 0 || (long long)n * D >= (1LL << 31)) return HD_ERR_UNSUPPORTED;
   if (!aligned16(workspace) || workspace_bytes < need) return HD_ERR_WORKSPACE;
-  return cuda_status(hdsfa::launch_expand_bwd(dout, ids, dtables, B, L, n, V, D, workspace, dev_status, stream));
+  hd_status_t st = hd_expand_embed_bwd_plan(ids, B, L, V, workspace, workspace_bytes, dev_status, stream);
+  if (st != HD_OK) return st;
+  return hd_expand_embed_bwd_apply(dout, dtables, B, L, n, V, D, workspace, workspace_bytes, stream);
 }
 
 hd_status_t hd_select_final_stream(const void* x, void* y, int B, int L, int n, int D, cudaStream_t stream) {

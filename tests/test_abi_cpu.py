@@ -94,9 +94,13 @@ def test_expand_validation(lib):
 
 
 def test_expand_bwd_workspace_size(lib):
-    assert lib.hd_expand_embed_bwd_workspace_bytes(1, 1) == 2048 * 8      # one shared-memory block of keys
-    assert lib.hd_expand_embed_bwd_workspace_bytes(1, 4096) == 4096 * 8
-    assert lib.hd_expand_embed_bwd_workspace_bytes(3, 1500) == 8192 * 8   # next power of two
+    # sorted keys (u64, padded to a power of two, at least one 4096-key block), two
+    # run lists of 16-byte records, one per token, two counters (16 bytes), and up to
+    # 16384 tokens the rank counts, one u64 per token and 256-key tile
+    assert lib.hd_expand_embed_bwd_workspace_bytes(1, 1) == 4096 * 8 + 2 * 16 + 16 + 8
+    assert lib.hd_expand_embed_bwd_workspace_bytes(1, 4096) == 4096 * 8 + 2 * 4096 * 16 + 16 + 16 * 4096 * 8
+    assert lib.hd_expand_embed_bwd_workspace_bytes(3, 1500) == 8192 * 8 + 2 * 4500 * 16 + 16 + 18 * 4500 * 8
+    assert lib.hd_expand_embed_bwd_workspace_bytes(4, 4500) == 32768 * 8 + 2 * 18000 * 16 + 16  # bitonic
     assert lib.hd_expand_embed_bwd_workspace_bytes(0, 4) == 0
     assert lib.hd_expand_embed_bwd_workspace_bytes(1 << 16, 1 << 15) == 0  # B*L must stay below 2^31
 
@@ -116,6 +120,18 @@ def test_expand_bwd_validation(lib):
     assert call(wb=ws - 8) == 4                # workspace too small
     assert call(w=0) == 4
     assert call(n=1 << 20, D=1 << 12) == 2     # n*D beyond 2^31
+
+
+def test_expand_bwd_plan_apply_validation(lib):
+    P, Z = ctypes.c_void_p, ctypes.c_size_t
+    ws = lib.hd_expand_embed_bwd_workspace_bytes(1, 4)
+    assert lib.hd_expand_embed_bwd_plan(None, 1, 4, 16, P(FAKE), Z(ws), None, None) == 1
+    assert lib.hd_expand_embed_bwd_plan(P(FAKE), 1, 4, 0, P(FAKE), Z(ws), None, None) == 1
+    assert lib.hd_expand_embed_bwd_plan(P(FAKE), 1, 4, 16, P(FAKE), Z(ws - 1), None, None) == 4
+    assert lib.hd_expand_embed_bwd_plan(P(FAKE), 1, 4, 16, P(FAKE + 8), Z(ws), None, None) == 4
+    assert lib.hd_expand_embed_bwd_apply(P(FAKE), P(FAKE), 1, 4, 2, 16, 12, P(FAKE), Z(ws), None) == 1
+    assert lib.hd_expand_embed_bwd_apply(P(FAKE), P(FAKE), 1, 4, 2, 16, 16, P(FAKE), Z(ws - 1), None) == 4
+    assert lib.hd_expand_embed_bwd_apply(P(FAKE), P(FAKE + 4), 1, 4, 2, 16, 16, P(FAKE), Z(ws), None) == 1
 
 
 def test_select_final_validation(lib):

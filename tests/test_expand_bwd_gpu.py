@@ -4,8 +4,9 @@ selection the loss reads (Eq. 2) with its adjoint, against the oracle.
 Selection and its adjoint are bit copies: bit-exact.  The expansion backward sums
 bf16 rows in fp32; the fp64 oracle differs from it only by rounding, bounded per
 element by (m + 1) * 2^-24 * (sum of |terms| + |initial value|) with m the largest
-number of occurrences of one id (sequential fp32 summation).  The kernel's sums are
-also checked bitwise for repeatability."""
+number of occurrences of one id (the bound of sequential fp32 summation, which also
+covers the kernel's blocked order for long runs).  The kernel's sums are also
+checked bitwise for repeatability."""
 import pytest
 import torch
 
@@ -63,7 +64,9 @@ def test_tiny_config():
     (2, 129, 3, 300, 136, 0.0),      # odd n, ragged slice of chunks
     (1, 1, 8, 5, 64, 0.0),           # one token
     (2, 513, 4, 64, 1024, 0.0),      # ~16 occurrences of every id
-    (1, 5000, 2, 37, 64, 0.0),       # keys beyond one shared-memory block: global sort steps
+    (1, 5000, 2, 37, 64, 0.0),       # 5000 tokens: sorted by rank count (20 x 20 tiles)
+    (4, 4500, 1, 3000, 64, 1.0),     # 18000 tokens: bitonic sort, global steps past 4096 keys
+    (1, 16384, 1, 700, 16, 0.0),     # the largest batch sorted by rank count
     (4, 1500, 4, 20000, 512, 1.1),   # Zipf ids: long runs of the frequent ids
 ])
 def test_shapes_accumulate(B, L, n, V, D, zipf):
@@ -81,6 +84,50 @@ def test_single_id_repeated_everywhere():
     got = _gpu_expand_bwd(dX, ids, n, V)
     _check_sum(got, dX, ids, n, V)
     assert torch.count_nonzero(got[:, :7]) == 0 and torch.count_nonzero(got[:, 8:]) == 0
+
+
+def test_run_lengths_around_the_split():
+    # ids occurring 31, 32, 33, 64 and 257 times (runs up to 32 tokens are summed in token
+    # order, longer ones in eight token blocks), plus 100 other tokens, shuffled
+    counts = {5: 31, 6: 32, 7: 33, 8: 64, 9: 257}
+    gen = torch.Generator().manual_seed(4)
+    rest = torch.randint(10, 500, (100,), generator=gen)
+    flat = torch.cat([torch.full((c,), v) for v, c in counts.items()] + [rest])
+    flat = flat[torch.randperm(flat.numel(), generator=gen)]
+    B, n, V, D = 1, 2, 500, 128
+    ids = flat.view(B, -1).to(torch.int32)
+    L = ids.shape[1]
+    dX = inputs.normal_bf16((B, n * L, D), seed=13)
+    dE0 = inputs.normal_bf16((n, V, D), seed=14).float()
+    _check_sum(_gpu_expand_bwd(dX, ids, n, V, dE0), dX, ids, n, V, dE0)
+
+
+def test_plan_once_apply_twice_on_another_stream():
+    # a plan built on a side stream, applied (after an event) to two different gradients
+    B, L, n, V, D = 2, 700, 4, 300, 256
+    ids = inputs.token_ids(B, L, V, seed=15, zipf=1.0)
+    dX1 = inputs.normal_bf16((B, n * L, D), seed=16)
+    dX2 = inputs.normal_bf16((B, n * L, D), seed=17)
+    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device="cuda")
+    side = torch.cuda.Stream()
+    idd = ids.cuda()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(side):
+        binding.hd_expand_embed_bwd_plan(idd, V, ws, stream=side)
+        done = torch.cuda.Event()
+        done.record(side)
+    torch.cuda.current_stream().wait_event(done)
+    dE = torch.zeros(n, V, D, dtype=torch.float32, device="cuda")
+    binding.hd_expand_embed_bwd_apply(dX1.cuda(), dE, ws, L)
+    torch.cuda.synchronize()
+    _check_sum(dE.cpu(), dX1, ids, n, V)
+    dE2 = torch.zeros(n, V, D, dtype=torch.float32, device="cuda")
+    binding.hd_expand_embed_bwd_apply(dX2.cuda(), dE2, ws, L)
+    torch.cuda.synchronize()
+    _check_sum(dE2.cpu(), dX2, ids, n, V)
+    # plan + apply gives the one-call result bit for bit
+    one = _gpu_expand_bwd(dX2, ids, n, V)
+    assert torch.equal(one.view(torch.int32), dE2.cpu().view(torch.int32))
 
 
 def test_deterministic_bits():
