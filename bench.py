@@ -303,56 +303,48 @@ def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2, window: int =
 
 
 # ---------------------------------------------------------------- bandwidth ops
-_FLUSH = None
+def time_op(fn, sets: int, iters=21, warmup=3):
+    """Device time (s) per call of fn(k), k = call index: `iters` calls back to back
+    between two events, the call k using buffer set k % sets (sets chosen so that
+    consecutive calls touch more than the 129 MB L2 and read from HBM)."""
+    for k in range(warmup):
+        fn(k % sets)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for k in range(iters):
+        fn(k % sets)
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / 1e3 / iters
 
 
-def flush_l2(dev):
-    """Overwrite a 256 MB buffer (twice the 129 MB L2) so the next launch reads from HBM."""
-    global _FLUSH
-    if _FLUSH is None:
-        _FLUSH = torch.empty(64 << 20, dtype=torch.float32, device=dev)
-    _FLUSH.fill_(1.0)
-
-
-def time_op(fn, dev, iters=10, warmup=3):
-    """Median device time (s) of fn(), each call timed alone after an L2 flush."""
-    for _ in range(warmup):
-        fn()
-    ts = []
-    for _ in range(iters):
-        flush_l2(dev)
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
-        fn()
-        b.record()
-        torch.cuda.synchronize()
-        ts.append(a.elapsed_time(b) / 1e3)
-    return statistics.median(ts)
-
-
-def measure_expansion_backward(dev, hbm_peak: float):
+def measure_expansion_backward(dev, hbm_peak: float, V: int = GATHER_V):
     """Expansion backward (adjoint of Eq. 1) and final-stream selection (Eq. 2) with
     its adjoint at the step's shapes: L=4096 tokens, n=4, D=4096, V=151936.
     Algorithmic bytes: expansion backward reads dX (n*L*D bf16) and the ids and
     reads + writes the fp32 rows of the distinct ids (U*n*D*8); its apply part (the
     row sums after the id-only plan) the same without the ids; selection reads and
-    writes L*D bf16; its adjoint reads L*D and writes n*L*D bf16."""
+    writes L*D bf16; its adjoint reads L*D and writes n*L*D bf16.  Three buffer sets
+    rotate so that no call finds its inputs in L2."""
     from paper_2607_08186_gb300 import binding, inputs
-    B, L, n, V, D = 1, 4096, 4, GATHER_V, GATHER_D
+    B, L, n, D = 1, 4096, 4, GATHER_D
+    S = 3
     g = torch.Generator(device=dev)
     g.manual_seed(31)
-    dX = torch.randn(B, n * L, D, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    dX = [torch.randn(B, n * L, D, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+          for _ in range(S)]
     dE = torch.zeros(n, V, D, dtype=torch.float32, device=dev)
     ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device=dev)
     out = {}
     for name, zipf in (("uniform_ids", 0.0), ("zipf1_ids", 1.0)):
         ids = inputs.token_ids(B, L, V, seed=31, zipf=zipf).to(dev)
         U = int(torch.unique(ids).numel())
-        t = time_op(lambda: binding.hd_expand_embed_bwd(dX, ids, dE, ws), dev)
+        t = time_op(lambda k: binding.hd_expand_embed_bwd(dX[k], ids, dE, ws), S)
         nbytes = B * n * L * D * 2 + B * L * 4 + U * n * D * 8
         binding.hd_expand_embed_bwd_plan(ids, V, ws)
-        t_apply = time_op(lambda: binding.hd_expand_embed_bwd_apply(dX, dE, ws, L), dev)
-        t_plan = time_op(lambda: binding.hd_expand_embed_bwd_plan(ids, V, ws), dev)
+        t_apply = time_op(lambda k: binding.hd_expand_embed_bwd_apply(dX[k], dE, ws, L), S)
+        t_plan = time_op(lambda k: binding.hd_expand_embed_bwd_plan(ids, V, ws), S)
         ab = nbytes - B * L * 4
         out[f"expand_bwd_{name}"] = {"ms": t * 1e3, "distinct_ids": U, "bytes": nbytes,
                                      "gbs": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / hbm_peak,
@@ -360,16 +352,17 @@ def measure_expansion_backward(dev, hbm_peak: float):
                                      "apply_gbs": ab / t_apply / 1e9,
                                      "apply_frac_hbm": ab / t_apply / 1e9 / hbm_peak}
     del dE
-    y = torch.empty(B, L, D, dtype=torch.bfloat16, device=dev)
-    t = time_op(lambda: binding.hd_select_final_stream(dX, y, n), dev)
+    y = [torch.empty(B, L, D, dtype=torch.bfloat16, device=dev) for _ in range(S)]
+    t = time_op(lambda k: binding.hd_select_final_stream(dX[k], y[k], n), S)
     nbytes = 2 * B * L * D * 2
     out["select_final"] = {"ms": t * 1e3, "bytes": nbytes, "gbs": nbytes / t / 1e9,
                            "frac_hbm": nbytes / t / 1e9 / hbm_peak}
-    t = time_op(lambda: binding.hd_select_final_stream_bwd(y, dX, n), dev)
+    t = time_op(lambda k: binding.hd_select_final_stream_bwd(y[k], dX[k], n), S)
     nbytes = B * L * D * 2 + B * n * L * D * 2
     out["select_final_bwd"] = {"ms": t * 1e3, "bytes": nbytes, "gbs": nbytes / t / 1e9,
                                "frac_hbm": nbytes / t / 1e9 / hbm_peak}
-    out["workload"] = f"B={B} L={L} n={n} V={V} D={D}, inputs flushed from L2 before each launch"
+    out["workload"] = (f"B={B} L={L} n={n} V={V} D={D}; 21 calls back to back over {S} rotating "
+                       "buffer sets (no call finds its inputs in L2)")
     del dX, y, ws
     torch.cuda.empty_cache()
     return out
@@ -480,6 +473,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-extras", action="store_true", help="skip the extras (CROSS / LOCAL layers, n sweep, expansion backward) and the CPU baseline")
+    ap.add_argument("--expand-bwd-only", action="store_true",
+                    help="time only the expansion backward and final-stream selection (JSON line)")
+    ap.add_argument("--vocab", type=int, default=GATHER_V,
+                    help="table rows V for --expand-bwd-only (smaller V for traffic captures)")
     ap.add_argument("--layer-only", choices=["within", "cross", "local"], default=None,
                     help="time only one attention layer (fwd + bwd, no gather / e2e / extras); "
                          "the small case used for kernel profiles")
@@ -499,6 +496,11 @@ def main():
     barrier(ws)
     s = SHAPES[WORKLOAD]
     pk = peaks()
+    if args.expand_bwd_only:
+        r = measure_expansion_backward(dev, pk["hbm"], V=args.vocab)
+        if rank == 0:
+            print(json.dumps(r), flush=True)
+        return
     if args.layer_only:
         mode = {"within": WITHIN, "cross": CROSS, "local": LOCAL}[args.layer_only]
         w = 4096 if mode == LOCAL else 0

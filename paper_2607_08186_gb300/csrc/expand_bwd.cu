@@ -137,6 +137,7 @@ __global__ void __launch_bounds__(256) scatter_kernel(const int32_t* __restrict_
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= N) return;
   unsigned long long acc = 0;  // fields stay below 2^15 (N <= kRankMax): no carries
+#pragma unroll 8
   for (int y = 0; y < tiles; ++y) acc += partial[(long long)y * N + i];
   const unsigned mask = (1u << kField) - 1;
   const unsigned r = (unsigned)acc & mask, m = (unsigned)(acc >> kField) & mask;
