@@ -81,6 +81,11 @@ def _load():
             lib.hdo_sfa_bwd_kv_rows.argtypes = [P, P, P, P, P, P, D, I64, P, P, P]
             lib.hdo_sfa_bwd.argtypes = [P, P, P, P, P, P, P, P, P, D]
             lib.hdo_sfa_bwd_jacobian.argtypes = [P, P, P, P, P, P, P, D]
+            lib.hdo_decode.restype = I64
+            lib.hdo_decode.argtypes = [P, P, P, P, P, P, I64, I64, I64, I64, I64, I64, ctypes.c_double,
+                                       ctypes.c_int, I64]
+            lib.hdo_kv_append.restype = I64
+            lib.hdo_kv_append.argtypes = [P, P, P, I64, I64, I64, I64]
             lib.hdo_num_threads.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -170,6 +175,40 @@ def select_final_bwd(dY: torch.Tensor, n: int):
     out = np.empty((B, n * L, D), dtype=np.uint16)
     _load().hdo_select_final_bwd(_ptr(yb), _ptr(out), B, L, n, D)
     return torch.from_numpy(out.view(np.int16)).view(torch.bfloat16)
+
+
+def decode(q, k_cache, v_cache, lens, n: int, mode: int, scale: float | None = None, window: int = 0):
+    """Decoding step over the expanded KV cache (Sec. 3.2 "Inference Cost"): the new
+    token's n positions attend under the layer's mask to the lens[b] * n cached positions.
+    q [B][n][Hq][Dh]; k_cache / v_cache [B][Lcap*n][Hkv][Dh]; lens [B] tokens in the cache
+    (new token included).  Returns (O fp64 [B][n][Hq][Dh], LSE fp64 [B][Hq][n], number of
+    sequences with lens outside [1, Lcap], which get zero rows and LSE = -inf)."""
+    qa, ka, va = _f64(q), _f64(k_cache), _f64(v_cache)
+    B, nq, Hq, Dh = qa.shape
+    if nq != n or ka.shape[1] % n:
+        raise ValueError("bad shapes")
+    Lcap, Hkv = ka.shape[1] // n, ka.shape[2]
+    if scale is None or scale <= 0:
+        scale = 1.0 / float(Dh) ** 0.5
+    la = np.ascontiguousarray(torch.as_tensor(lens).to(torch.int32).cpu().numpy())
+    o = np.empty_like(qa)
+    lse = np.empty((B, Hq, n))
+    bad = _load().hdo_decode(_ptr(qa), _ptr(ka), _ptr(va), _ptr(la), _ptr(o), _ptr(lse), B, Lcap, n, Hq,
+                             Hkv, Dh, float(scale), int(mode), int(window))
+    return torch.from_numpy(o), torch.from_numpy(lse), int(bad)
+
+
+def kv_append(new_rows, cache, lens, n: int):
+    """The new token's n K (or V) rows into the cache at positions (lens[b]-1)*n + s,
+    on bf16 bit patterns.  new_rows [B][n][Hkv][Dh], cache [B][Lcap*n][Hkv][Dh] (a copy is
+    returned).  Returns (cache', number of sequences with lens outside [1, Lcap])."""
+    B, nn, Hkv, Dh = new_rows.shape
+    Lcap = cache.shape[1] // n
+    nb = np.ascontiguousarray(new_rows.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16))
+    cb = np.ascontiguousarray(cache.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)).copy()
+    la = np.ascontiguousarray(torch.as_tensor(lens).to(torch.int32).cpu().numpy())
+    bad = _load().hdo_kv_append(_ptr(nb), _ptr(cb), _ptr(la), B, Lcap, n, Hkv * Dh)
+    return torch.from_numpy(cb.view(np.int16)).view(torch.bfloat16), int(bad)
 
 
 def sfa_fwd(q, k, v, n: int, mode: int, scale: float | None = None, window: int = 0):

@@ -13,6 +13,9 @@
  *              its adjoint (the gradient with respect to the n tables).
  *   - Eq. 2  : the final-stream positions t = i n that the loss reads, and their
  *              adjoint.
+ *   - Sec. 3.2 "Inference Cost": decoding, where each new token's n positions
+ *              attend to the expanded KV cache (the forward's rows for that token),
+ *              and the cache append of the new token's n K/V rows.
  *   - Eq. 3  : token index i(t) = ceil(t/n) and stream index s(t) = ((t-1) mod n) + 1.
  *   - Eq. 4  : the intra-stream mask M[t,t'] = 1[t' <= t and s(t') = s(t)] (WITHIN).
  *   - Fig. 2a: the full cross-stream layer, the standard causal mask over all
@@ -168,6 +171,81 @@ static double row_scores(const double* q, const double* k, const hdo_dims* d,
   for (int64_t pk = 0; pk < nL; ++pk)
     if (vis0(d, p, pk)) sum += exp(z[pk] - m);
   return m + log(sum);
+}
+
+/* ---- Decoding with the expanded KV cache (Sec. 3.2 "Inference Cost") ----
+ * Generation processes each new token's n streams together in one forward pass.
+ * With i = lens[b] tokens of sequence b in the cache (the new token i included, its
+ * K/V already stored), the new token's positions t = (i-1)n + k, k = 1..n, attend
+ * under the layer's mask (Eq. 4, Fig. 2) to the cached positions 1 .. i n: the same
+ * masked softmax attention as the forward, for the new token's rows only.  Intra-stream
+ * layers thus read only their own stream's cached keys; cross-stream layers read all.
+ *   q, o   : [B][n][Hq][Dh] (row k-1 = stream k of the new token)
+ *   kc, vc : [B][Lcap n][Hkv][Dh] (position t at row t-1)
+ *   lens   : [B], tokens in the cache, valid in [1, Lcap]
+ *   lse    : [B][Hq][n] natural log
+ * A sequence whose lens is outside [1, Lcap] gets zero rows and lse = -inf; the
+ * return value counts such sequences. */
+int64_t hdo_decode(const double* q, const double* kc, const double* vc, const int32_t* lens, double* o,
+                   double* lse, int64_t B, int64_t Lcap, int64_t n, int64_t Hq, int64_t Hkv, int64_t Dh,
+                   double scale, int mode, int64_t window) {
+  int64_t bad = 0;
+  for (int64_t b = 0; b < B; ++b) {
+    const int64_t i = lens[b];
+    const int valid = i >= 1 && i <= Lcap;
+    if (!valid) ++bad;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t k = 1; k <= n; ++k) {
+      for (int64_t h = 0; h < Hq; ++h) {
+        const double* qr = q + ((b * n + (k - 1)) * Hq + h) * Dh;
+        double* orow = o + ((b * n + (k - 1)) * Hq + h) * Dh;
+        double* l = lse + (b * Hq + h) * n + (k - 1);
+        for (int64_t e = 0; e < Dh; ++e) orow[e] = 0.0;
+        if (!valid) {
+          *l = -INFINITY;
+          continue;
+        }
+        const int64_t t = (i - 1) * n + k, g = h / (Hq / Hkv);
+        double m = -INFINITY;
+        for (int64_t tk = 1; tk <= i * n; ++tk) {
+          if (!hdo_visible(t, tk, n, mode, window)) continue;
+          const double z = scale * dot(qr, kc + ((b * Lcap * n + tk - 1) * Hkv + g) * Dh, Dh);
+          if (z > m) m = z;
+        }
+        double sum = 0.0;
+        for (int64_t tk = 1; tk <= i * n; ++tk) {
+          if (!hdo_visible(t, tk, n, mode, window)) continue;
+          const double z = scale * dot(qr, kc + ((b * Lcap * n + tk - 1) * Hkv + g) * Dh, Dh);
+          const double w = exp(z - m);
+          sum += w;
+          const double* vr = vc + ((b * Lcap * n + tk - 1) * Hkv + g) * Dh;
+          for (int64_t e = 0; e < Dh; ++e) orow[e] += w * vr[e];
+        }
+        for (int64_t e = 0; e < Dh; ++e) orow[e] /= sum;
+        *l = m + log(sum);
+      }
+    }
+  }
+  return bad;
+}
+
+/* The new token's K (or V) rows enter the cache at its n positions:
+ * cache[b][(i-1)n + k - 1] = new[b][k-1] with i = lens[b] (bf16 bit patterns, rows of
+ * Hkv*Dh).  Sequences with lens outside [1, Lcap] are left untouched (counted). */
+int64_t hdo_kv_append(const uint16_t* nw, uint16_t* cache, const int32_t* lens, int64_t B, int64_t Lcap,
+                      int64_t n, int64_t row) {
+  int64_t bad = 0;
+  for (int64_t b = 0; b < B; ++b) {
+    const int64_t i = lens[b];
+    if (i < 1 || i > Lcap) {
+      ++bad;
+      continue;
+    }
+    for (int64_t k = 1; k <= n; ++k)
+      memcpy(cache + (b * Lcap * n + (i - 1) * n + k - 1) * row, nw + (b * n + k - 1) * row,
+             (size_t)row * sizeof(uint16_t));
+  }
+  return bad;
 }
 
 /* ---- forward for one row: O[b,p,h] = sum_p' P[p,p'] V[p'], P = softmax over visible keys */

@@ -441,3 +441,83 @@ def test_bwd_row_functions_match_full():
         for r, (b, g, p) in enumerate(kvrows):
             torch.testing.assert_close(dkr[r], dk[b, p, g], rtol=1e-12, atol=1e-13)
             torch.testing.assert_close(dvr[r], dv[b, p, g], rtol=1e-12, atol=1e-13)
+
+
+# ------------------------------------------------------------------ decoding (Sec. 3.2)
+@pytest.mark.parametrize("n", [1, 2, 4])
+@pytest.mark.parametrize("mode,w", [(oracle.WITHIN, 0), (oracle.CROSS, 0), (oracle.LOCAL, 5)])
+def test_decode_is_forward_rows_of_the_last_token(n, mode, w):
+    # decoding token i with the cache holding tokens 1..i equals the forward pass's rows
+    # of token i; a shorter sequence (lens < Lcap) equals the forward over its prefix
+    B, L, Hq, Hkv, Dh, scale = 2, 7, 4, 2, 16, 0.35
+    q, k, v = _rand((B, n * L, Hq, Dh), 40), _rand((B, n * L, Hkv, Dh), 41), _rand((B, n * L, Hkv, Dh), 42)
+    lens = torch.tensor([L, 3], dtype=torch.int32)
+    qn = torch.stack([q[b, (int(lens[b]) - 1) * n:int(lens[b]) * n] for b in range(B)])
+    o, lse, bad = oracle.decode(qn, k, v, lens, n, mode, scale, window=w)
+    assert bad == 0
+    for b in range(B):
+        i = int(lens[b])
+        of, lf = oracle.sfa_fwd(q[b:b + 1, :i * n], k[b:b + 1, :i * n], v[b:b + 1, :i * n], n, mode, scale,
+                                window=w)
+        torch.testing.assert_close(o[b], of[0, (i - 1) * n:i * n], rtol=1e-12, atol=1e-12)
+        torch.testing.assert_close(lse[b], lf[0, :, (i - 1) * n:i * n], rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("mode", [oracle.WITHIN, oracle.CROSS])
+def test_decode_matches_masked_sdpa(mode):
+    # torch fp64 SDPA of the new token's n query rows against all cached rows under an
+    # explicit boolean mask (0-indexed: key p' visible from p = (i-1)n + s iff p' <= p,
+    # and for the intra-stream layer p' = s mod n)
+    B, n, Lcap, Hq, Hkv, Dh, scale = 1, 3, 10, 6, 2, 8, 0.5
+    i = 8
+    kc, vc = _rand((B, n * Lcap, Hkv, Dh), 43), _rand((B, n * Lcap, Hkv, Dh), 44)
+    qn = _rand((B, n, Hq, Dh), 45)
+    o, _, _ = oracle.decode(qn, kc, vc, torch.tensor([i], dtype=torch.int32), n, mode, scale)
+    p = (i - 1) * n + torch.arange(n)
+    pk = torch.arange(i * n)
+    mask = pk[None, :] <= p[:, None]
+    if mode == oracle.WITHIN:
+        mask &= (pk[None, :] % n) == (p[:, None] % n)
+    qh = qn.permute(0, 2, 1, 3)
+    kh = kc[:, :i * n].permute(0, 2, 1, 3).repeat_interleave(Hq // Hkv, dim=1)
+    vh = vc[:, :i * n].permute(0, 2, 1, 3).repeat_interleave(Hq // Hkv, dim=1)
+    ref = F.scaled_dot_product_attention(qh, kh, vh, attn_mask=mask, scale=scale).permute(0, 2, 1, 3)
+    torch.testing.assert_close(o, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_decode_n1_is_single_query_attention():
+    # n = 1: one query per step attending to every cached token (closed form softmax(qK^T)V)
+    B, Lcap, Hq, Hkv, Dh, scale = 2, 9, 2, 1, 8, 0.7
+    kc, vc, qn = _rand((B, Lcap, Hkv, Dh), 46), _rand((B, Lcap, Hkv, Dh), 47), _rand((B, 1, Hq, Dh), 48)
+    lens = torch.tensor([9, 4], dtype=torch.int32)
+    o, lse, _ = oracle.decode(qn, kc, vc, lens, 1, oracle.CROSS, scale)
+    for b in range(B):
+        i = int(lens[b])
+        z = scale * torch.einsum("hd,kd->hk", qn[b, 0], kc[b, :i, 0])
+        P = torch.softmax(z, dim=-1)
+        torch.testing.assert_close(o[b, 0], P @ vc[b, :i, 0], rtol=1e-12, atol=1e-12)
+        torch.testing.assert_close(lse[b, :, 0], torch.logsumexp(z, dim=-1), rtol=1e-12, atol=1e-12)
+
+
+def test_decode_bad_lens_zero_rows():
+    B, n, Lcap, H, Dh = 3, 2, 4, 2, 8
+    kc, vc, qn = _rand((B, n * Lcap, H, Dh), 49), _rand((B, n * Lcap, H, Dh), 50), _rand((B, n, H, Dh), 51)
+    lens = torch.tensor([0, 4, 5], dtype=torch.int32)
+    o, lse, bad = oracle.decode(qn, kc, vc, lens, n, oracle.CROSS)
+    assert bad == 2
+    assert torch.count_nonzero(o[0]) == 0 and torch.count_nonzero(o[2]) == 0
+    assert torch.isinf(lse[0]).all() and torch.isinf(lse[2]).all() and torch.isfinite(lse[1]).all()
+
+
+def test_kv_append_matches_indexing():
+    B, n, Lcap, Hkv, Dh = 3, 4, 5, 2, 8
+    cache = _rand((B, n * Lcap, Hkv, Dh), 52, torch.bfloat16)
+    new = _rand((B, n, Hkv, Dh), 53, torch.bfloat16)
+    lens = torch.tensor([1, 5, 7], dtype=torch.int32)     # the last is out of range
+    got, bad = oracle.kv_append(new, cache, lens, n)
+    assert bad == 1
+    ref = cache.clone()
+    for b in range(2):
+        i = int(lens[b])
+        ref[b, (i - 1) * n:i * n] = new[b]
+    assert torch.equal(got.view(torch.int16), ref.view(torch.int16))
