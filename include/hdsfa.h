@@ -46,7 +46,8 @@ typedef enum {
 
 /* Bits the kernels OR into *dev_status. */
 #define HD_DEVBIT_INDEX 1   /* a token id outside [0, V): hd_expand_embed zeroed its n output
-                               rows; hd_expand_embed_bwd left it out of the sums */
+                               rows; hd_expand_embed_bwd left it out of the sums.  A sequence
+                               length outside its range in sfa_decode / sfa_kv_append */
 #define HD_DEVBIT_TIMEOUT 2 /* a bounded pipeline wait expired; outputs are invalid */
 
 /* Attention mask of one SFA layer (Sec. 2.2, Eq. 4 and Fig. 2). */
@@ -174,6 +175,46 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
 hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
                              float softmax_scale, sfa_mode_t mode, void* workspace,
                              size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * sfa_decode -- one decoding step over the expanded KV cache (Sec. 3.2 "Inference
+ * Cost"; masks of Eq. 4 and Fig. 2).  Generation runs each new token's n streams
+ * together: with T = lens[b] tokens in sequence b's cache (the new token included,
+ * its K/V rows already appended, see sfa_kv_append), the new token's positions
+ * p = (T-1)*n + s attend to the cached positions p' < T*n that the layer's mask lets
+ * them see: WITHIN p' = s (mod n) and p' <= p (only stream s's rows are read for it),
+ * CROSS p' <= p, LOCAL p - window < p' <= p.  The result equals rows (T-1)*n .. T*n-1
+ * of sfa_fwd over the sequence.
+ *   q, o     : bf16 [B][n][Hq][Dh], the new token's n positions.
+ *   k_cache, v_cache : bf16 [B][Lcap*n][Hkv][Dh], position p at row p (the layout of
+ *              sfa_fwd's k / v, so a prefilled forward's K/V is a cache); read-only.
+ *   lens     : int32 device array [B], tokens in each sequence's cache (ragged batch).
+ *   lse      : float32 [B][Hq][n] natural-log LSE of each row, or NULL.
+ *   max_tokens: a bound on every lens[b] (<= Lcap); the work is split for it.
+ *   workspace: device memory of >= sfa_decode_workspace_bytes(B, max_tokens, n, Hq,
+ *              Hkv, Dh, mode, window) bytes, 16-byte aligned (partial results).
+ * A sequence with lens outside [1, max_tokens] gets zero rows, LSE = -inf and
+ * HD_DEVBIT_INDEX.  Dh in {64, 128}; Lcap*n <= 2^30.  HBM-bound (reads the visible
+ * cached rows once per step).
+ */
+size_t sfa_decode_workspace_bytes(int B, int max_tokens, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode,
+                                  int window); /* 0 for invalid sizes */
+hd_status_t sfa_decode(const void* q, const void* k_cache, const void* v_cache, const int32_t* lens, void* o,
+                       float* lse, int B, int max_tokens, int Lcap, int n, int Hq, int Hkv, int Dh,
+                       float softmax_scale, sfa_mode_t mode, int window, void* workspace,
+                       size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream);
+
+/*
+ * sfa_kv_append -- the new token's n K and V rows into the cache (Sec. 3.2: each
+ * decoded token adds n stream positions):
+ *   k_cache[b][(T-1)*n + s] = k_new[b][s], likewise v, with T = lens[b] (the length
+ *   including the new token), s < n.
+ *   k_new, v_new: bf16 [B][n][Hkv][Dh]; caches as in sfa_decode.  Bit copy.
+ * A length outside [1, Lcap] writes nothing for that sequence and sets HD_DEVBIT_INDEX.
+ */
+hd_status_t sfa_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache,
+                          const int32_t* lens, int B, int Lcap, int n, int Hkv, int Dh,
+                          int32_t* dev_status, cudaStream_t stream);
 
 /*
  * sfa_bwd_noalloc -- sfa_bwd without a caller-supplied workspace.  The paper has no

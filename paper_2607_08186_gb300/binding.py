@@ -55,6 +55,12 @@ def lib():
             L.hd_select_final_stream.argtypes = [P, P, I, I, I, I, P]
             L.hd_select_final_stream_bwd.restype = I
             L.hd_select_final_stream_bwd.argtypes = [P, P, I, I, I, I, P]
+            L.sfa_decode_workspace_bytes.restype = Z
+            L.sfa_decode_workspace_bytes.argtypes = [I, I, I, I, I, I, I, I]
+            L.sfa_decode.restype = I
+            L.sfa_decode.argtypes = [P, P, P, P, P, P, I, I, I, I, I, I, I, F, I, I, P, Z, P, P]
+            L.sfa_kv_append.restype = I
+            L.sfa_kv_append.argtypes = [P, P, P, P, P, I, I, I, I, I, P, P]
             L.sfa_fwd.restype = I
             L.sfa_fwd.argtypes = [P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, P]
             L.sfa_bwd_workspace_bytes.restype = Z
@@ -192,6 +198,37 @@ def sfa_bwd(q, k, v, o, lse, dout, dq, dk, dv, n, mode, workspace, softmax_scale
                          _p(workspace), _wsb(workspace),
                          _p(dev_status), _stream(stream)), "sfa_bwd")
     return dq, dk, dv
+
+
+def sfa_decode_workspace_bytes(B, max_tokens, n, Hq, Hkv, Dh, mode, window=0) -> int:
+    return int(lib().sfa_decode_workspace_bytes(B, max_tokens, n, Hq, Hkv, Dh, int(mode), int(window)))
+
+
+def sfa_decode(q, k_cache, v_cache, lens, o, n, mode, workspace, max_tokens=None, lse=None, softmax_scale=0.0,
+               window=0, dev_status=None, stream=None):
+    """One decoding step (Sec. 3.2): the new token's n positions q [B][n][Hq][Dh] against
+    the cache k_cache / v_cache [B][Lcap*n][Hkv][Dh] holding lens[b] tokens (int32 CUDA
+    tensor [B]); o [B][n][Hq][Dh] bf16, lse [B][Hq][n] float32 or None.  max_tokens bounds
+    every lens[b] (default: the cache capacity Lcap)."""
+    B, nq, Hq, Dh = q.shape
+    if nq != n or k_cache.shape[1] % n:
+        raise ValueError("q.shape[1] must be n and k_cache.shape[1] a multiple of n")
+    Lcap, Hkv = k_cache.shape[1] // n, k_cache.shape[2]
+    T = Lcap if max_tokens is None else int(max_tokens)
+    _check(lib().sfa_decode(_p(q), _p(k_cache), _p(v_cache), _p(lens), _p(o), _p(lse), B, T, Lcap, n, Hq, Hkv,
+                            Dh, float(softmax_scale), int(mode), int(window), _p(workspace), _wsb(workspace),
+                            _p(dev_status), _stream(stream)), "sfa_decode")
+    return o
+
+
+def sfa_kv_append(k_new, v_new, k_cache, v_cache, lens, n, dev_status=None, stream=None):
+    """k_cache[b][(lens[b]-1)*n + s] = k_new[b][s] (and v): the new token's n K/V rows."""
+    B, nn, Hkv, Dh = k_new.shape
+    if nn != n:
+        raise ValueError("k_new.shape[1] must be n")
+    Lcap = k_cache.shape[1] // n
+    _check(lib().sfa_kv_append(_p(k_new), _p(v_new), _p(k_cache), _p(v_cache), _p(lens), B, Lcap, n, Hkv, Dh,
+                               _p(dev_status), _stream(stream)), "sfa_kv_append")
 
 
 SFA_BWD_NOALLOC_MAX_BYTES = 64 << 20

@@ -16,6 +16,17 @@ cudaError_t launch_expand_bwd_apply(const void* dx, float* de, int B, int L, int
                                     cudaStream_t st);
 cudaError_t launch_select_final(const void* x, void* y, int B, int L, int n, int D, cudaStream_t st);
 cudaError_t launch_select_final_bwd(const void* dy, void* dx, int B, int L, int n, int D, cudaStream_t st);
+struct DecodePlan {
+  int G, M, ngroups, nsplit, chunk;
+  size_t part_o_bytes, part_ml_bytes;
+};
+DecodePlan decode_plan(int B, int maxT, int n, int Hq, int Hkv, int Dh, int mode, int window);
+size_t decode_ws_bytes(const DecodePlan& p);
+cudaError_t launch_sfa_decode(const void* q, const void* kc, const void* vc, const int32_t* lens, void* o,
+                              float* lse, int B, int maxT, int Lcap, int n, int Hq, int Hkv, int Dh, float scale,
+                              int mode, int window, void* ws, int32_t* status, cudaStream_t st);
+cudaError_t launch_kv_append(const void* kn, const void* vn, void* kc, void* vc, const int32_t* lens, int B,
+                             int Lcap, int n, int Hkv, int Dh, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
                               const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
@@ -265,6 +276,52 @@ hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, 
   if (st != HD_OK) return st;
   return sfa_bwd_finalize(dq, B, L, n, Hq, Hkv, Dh, softmax_scale, mode, workspace,
                           workspace_bytes, stream);
+}
+
+// Sizes of a decode step: max_tokens bounds every sequence's length and the cache
+// capacity Lcap bounds max_tokens.
+static hd_status_t decode_sizes(int B, int maxT, int Lcap, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode,
+                                int window) {
+  if (B <= 0 || maxT <= 0 || Lcap <= 0 || n <= 0 || Hq <= 0 || Hkv <= 0 || Dh <= 0) return HD_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0 || maxT > Lcap) return HD_ERR_INVALID_ARG;
+  if (mode != SFA_WITHIN && mode != SFA_CROSS && mode != SFA_LOCAL) return HD_ERR_INVALID_ARG;
+  if (mode == SFA_LOCAL && window <= 0) return HD_ERR_INVALID_ARG;
+  if (Dh != 64 && Dh != 128) return HD_ERR_UNSUPPORTED;
+  if ((long long)Lcap * n > (1LL << 30) || (long long)n * Hq > (1LL << 20)) return HD_ERR_UNSUPPORTED;
+  return HD_OK;
+}
+
+size_t sfa_decode_workspace_bytes(int B, int max_tokens, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode,
+                                  int window) {
+  if (decode_sizes(B, max_tokens, max_tokens, n, Hq, Hkv, Dh, mode, window) != HD_OK) return 0;
+  return hdsfa::decode_ws_bytes(hdsfa::decode_plan(B, max_tokens, n, Hq, Hkv, Dh, mode, window));
+}
+
+hd_status_t sfa_decode(const void* q, const void* k_cache, const void* v_cache, const int32_t* lens, void* o,
+                       float* lse, int B, int max_tokens, int Lcap, int n, int Hq, int Hkv, int Dh,
+                       float softmax_scale, sfa_mode_t mode, int window, void* workspace, size_t workspace_bytes,
+                       int32_t* dev_status, cudaStream_t stream) {
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(o)) return HD_ERR_INVALID_ARG;
+  if (lens == nullptr || (reinterpret_cast<uintptr_t>(lens) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  if (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  hd_status_t st = decode_sizes(B, max_tokens, Lcap, n, Hq, Hkv, Dh, mode, window);
+  if (st != HD_OK) return st;
+  const size_t need = sfa_decode_workspace_bytes(B, max_tokens, n, Hq, Hkv, Dh, mode, window);
+  if (!aligned16(workspace) || workspace_bytes < need) return HD_ERR_WORKSPACE;
+  return cuda_status(hdsfa::launch_sfa_decode(q, k_cache, v_cache, lens, o, lse, B, max_tokens, Lcap, n, Hq, Hkv,
+                                              Dh, resolve_scale(softmax_scale, Dh), (int)mode,
+                                              mode == SFA_LOCAL ? window : 0, workspace, dev_status, stream));
+}
+
+hd_status_t sfa_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache, const int32_t* lens,
+                          int B, int Lcap, int n, int Hkv, int Dh, int32_t* dev_status, cudaStream_t stream) {
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
+    return HD_ERR_INVALID_ARG;
+  if (lens == nullptr || (reinterpret_cast<uintptr_t>(lens) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  if (B <= 0 || Lcap <= 0 || n <= 0 || Hkv <= 0 || Dh <= 0 || Dh % 8 != 0) return HD_ERR_INVALID_ARG;
+  if ((long long)Lcap * n > (1LL << 30)) return HD_ERR_UNSUPPORTED;
+  return cuda_status(hdsfa::launch_kv_append(k_new, v_new, k_cache, v_cache, lens, B, Lcap, n, Hkv, Dh,
+                                             dev_status, stream));
 }
 
 const char* hd_status_string(hd_status_t s) {

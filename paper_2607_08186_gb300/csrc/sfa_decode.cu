@@ -1,0 +1,445 @@
+// Decoding over the expanded KV cache (Sec. 3.2 "Inference Cost").
+//
+// Generation feeds each new token's n streams through the model together: its n
+// positions p = (T-1)n + s (T = tokens in the cache, the new one included, whose K/V
+// rows are already stored) attend, under the layer's mask, to the cached positions
+// 0 .. Tn-1.  An intra-stream layer (Eq. 4) reads only stream s's cached rows for
+// the queries of stream s; a cross-stream layer (Fig. 2a) reads all of them; a local
+// one (Fig. 2b) the last `window` positions.  The cache has the training layout,
+// [B][Lcap*n][Hkv][Dh] with position p at row p, so the forward pass's K/V tensors
+// are a filled cache.
+//
+// Memory-bound: every step streams the visible cached rows of K and V once.  Per K/V
+// head the queries are the n streams x (Hq/Hkv) heads of the group, 16 to 32 rows (a
+// CTA takes up to 32; more rows take several CTAs): far below a tcgen05 tile, so the
+// contractions use warp-level mma.sync m16n8k16 (bf16, fp32 accumulate), which keeps
+// up with HBM.  Split over the cached positions (flash-decoding):
+//   decode_kernel : CTA (split c, K/V head x row group, sequence): a 3-stage cp.async
+//                   ring of 64-position K/V tiles; warp w takes keys [16w, 16w+16) of
+//                   each tile with its own online softmax; the 4 warps merge in shared
+//                   memory and write an unnormalised partial (O, running max, sum).
+//   combine_kernel: merges a row's partials, writes O (bf16) and the natural-log LSE.
+// Masking is per element (the new token's own positions, the stream condition of an
+// intra-stream layer, the window); rows past the group's query count and positions
+// past the sequence are zero-filled and masked.  A sequence whose length is outside
+// [1, max_tokens] gets zero rows, LSE = -inf and HD_DEVBIT_INDEX.
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace hdsfa {
+
+typedef __nv_bfloat16 bf16;
+
+namespace dec {
+constexpr int NT = 128;      // 4 warps
+constexpr int KT = 64;       // cached positions per pipeline stage
+constexpr int STAGES = 3;
+constexpr int RG = 32;       // query rows per CTA at most (two m16 tiles)
+constexpr int kMaxSplit = 128;
+constexpr int kTargetCtas = 152 * 4;
+
+struct DecodeArgs {
+  const bf16* q;        // [B][n][Hq][Dh]
+  const bf16* kc;       // [B][Lcap*n][Hkv][Dh]
+  const bf16* vc;
+  const int32_t* lens;  // [B] tokens in the cache
+  bf16* o;              // [B][n][Hq][Dh]
+  float* lse;           // [B][Hq][n] or null
+  float* part_o;        // [B][Hkv][ngroups][nsplit][RG][Dh]
+  float2* part_ml;      // [B][Hkv][ngroups][nsplit][RG]: (max in log2 units, sum)
+  int32_t* status;
+  int B, Lcap, maxT, n, Hq, Hkv, G, M, ngroups, nsplit, chunk, mode, window;
+  float scale_log2;
+};
+
+// Visible position range [lo, hi) of a sequence of T tokens (the new token's rows
+// see nothing outside it; per-row conditions are applied per element).
+HD_DEVINLINE void seq_range(const DecodeArgs& a, int T, int& lo, int& hi) {
+  hi = T * a.n;
+  lo = a.mode == SFA_LOCAL ? max(0, (T - 1) * a.n - a.window + 1) : 0;
+}
+
+template <int DH, int MT>
+__global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  bf16* sQ = reinterpret_cast<bf16*>(smem_raw);  // [MT*16][DH]
+  bf16* sK = sQ + MT * 16 * DH;                   // [STAGES][KT][DH]
+  bf16* sV = sK + STAGES * KT * DH;               // [STAGES][KT][DH]
+  constexpr int CPR = DH / 8;
+  const int c = blockIdx.x, g = blockIdx.y / a.ngroups, rg = blockIdx.y % a.ngroups, b = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g4 = lane >> 2, t4 = lane & 3;
+  const size_t pidx = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit + c;
+  float* po = a.part_o + pidx * RG * DH;
+  float2* pml = a.part_ml + pidx * RG;
+  const int T = a.lens[b];
+  int k0 = 0, k1 = 0;
+  if (T >= 1 && T <= a.maxT) {
+    int lo, hi;
+    seq_range(a, T, lo, hi);
+    k0 = lo + c * a.chunk;
+    k1 = min(k0 + a.chunk, hi);
+  }
+  if (k0 >= k1) {  // nothing of this sequence in this split: an empty partial
+    for (int i = tid; i < RG; i += NT) pml[i] = make_float2(-INFINITY, 0.f);
+    return;
+  }
+  const long long pbase = (long long)b * a.Lcap * a.n;  // cache row of position 0
+
+  // query rows of the group -> smem (rows past M zero-filled)
+  for (int i = tid; i < MT * 16 * CPR; i += NT) {
+    const int rr = i / CPR, cc = i % CPR, r = rg * RG + rr;
+    const bool ok = r < a.M;
+    const int s = ok ? r / a.G : 0, h = g * a.G + (ok ? r % a.G : 0);
+    cp_async_16(smem_u32(sQ + swz<DH>(rr, cc * 8)), a.q + (((long long)b * a.n + s) * a.Hq + h) * DH + cc * 8,
+                ok);
+  }
+  auto load_stage = [&](int st, int kp0) {
+    bf16* dK = sK + st * KT * DH;
+    bf16* dV = sV + st * KT * DH;
+    for (int i = tid; i < KT * CPR; i += NT) {
+      const int rr = i / CPR, cc = i % CPR, p = kp0 + rr;
+      const bool ok = p < k1;
+      const long long off = ((pbase + (ok ? p : k0)) * a.Hkv + g) * DH + cc * 8;
+      cp_async_16(smem_u32(dK + swz<DH>(rr, cc * 8)), a.kc + off, ok);
+      cp_async_16(smem_u32(dV + swz<DH>(rr, cc * 8)), a.vc + off, ok);
+    }
+  };
+  const int nsub = (k1 - k0 + KT - 1) / KT;
+  load_stage(0, k0);
+  cp_async_commit();
+  if (nsub > 1) load_stage(1, k0 + KT);
+  cp_async_commit();
+
+  // this thread's query rows: (mt, half) -> local row mt*16 + g4 + 8*half
+  int rs_[MT][2], rq[MT][2];  // stream of the row (-1: padding row) and its position
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+    for (int hf = 0; hf < 2; ++hf) {
+      const int r = rg * RG + mt * 16 + g4 + 8 * hf;
+      rs_[mt][hf] = r < a.M ? r / a.G : -1;
+      rq[mt][hf] = (T - 1) * a.n + (r < a.M ? r / a.G : 0);
+    }
+  float mx[MT][2], ls[MT][2], oacc[MT][DH / 8][4];
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) {
+    mx[mt][0] = mx[mt][1] = -INFINITY;
+    ls[mt][0] = ls[mt][1] = 0.f;
+#pragma unroll
+    for (int i = 0; i < DH / 8; ++i) oacc[mt][i][0] = oacc[mt][i][1] = oacc[mt][i][2] = oacc[mt][i][3] = 0.f;
+  }
+
+  for (int it = 0; it < nsub; ++it) {
+    cp_async_wait<STAGES - 2>();  // stage `it` has landed
+    __syncthreads();              // ... for every thread, and stage it-1 is no longer read
+    if (it + 2 < nsub) load_stage((it + 2) % STAGES, k0 + (it + 2) * KT);
+    cp_async_commit();
+    const bf16* cK = sK + (it % STAGES) * KT * DH;
+    const bf16* cV = sV + (it % STAGES) * KT * DH;
+
+    float sacc[MT][2][4];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) sacc[mt][j][0] = sacc[mt][j][1] = sacc[mt][j][2] = sacc[mt][j][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < DH / 16; ++kk) {
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4(smem_u32(cK + swz<DH>(warp * 16 + (lane & 7) + (lane >> 4) * 8, kk * 16 + ((lane >> 3) & 1) * 8)),
+              b0, b1, b2, b3);
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        uint32_t qa[4];
+        ldsm_x4(smem_u32(sQ + swz<DH>(mt * 16 + (lane & 15), kk * 16 + (lane >> 4) * 8)), qa[0], qa[1], qa[2],
+                qa[3]);
+        mma_bf16_16816(sacc[mt][0], qa, b0, b1);
+        mma_bf16_16816(sacc[mt][1], qa, b2, b3);
+      }
+    }
+    // mask + online softmax (log2 domain)
+    const int kb = k0 + it * KT + warp * 16;
+    int kp[2][2], kst[2][2];
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        kp[j][e] = kb + j * 8 + 2 * t4 + e;
+        kst[j][e] = a.mode == SFA_WITHIN ? kp[j][e] % a.n : 0;
+      }
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+      float tmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+#pragma unroll
+        for (int e4 = 0; e4 < 4; ++e4) {
+          const int hf = e4 >> 1, e = e4 & 1, p = kp[j][e], pq = rq[mt][hf];
+          bool vis = rs_[mt][hf] >= 0 && p < k1 && p <= pq;
+          if (a.mode == SFA_WITHIN) vis = vis && kst[j][e] == rs_[mt][hf];
+          if (a.mode == SFA_LOCAL) vis = vis && p > pq - a.window;
+          const float x = vis ? sacc[mt][j][e4] * a.scale_log2 : -INFINITY;
+          sacc[mt][j][e4] = x;
+          tmax[hf] = fmaxf(tmax[hf], x);
+        }
+      float corr[2], muse[2];
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        tmax[hf] = fmaxf(tmax[hf], __shfl_xor_sync(0xffffffffu, tmax[hf], 1));
+        tmax[hf] = fmaxf(tmax[hf], __shfl_xor_sync(0xffffffffu, tmax[hf], 2));
+        const float mnew = fmaxf(mx[mt][hf], tmax[hf]);
+        muse[hf] = mnew == -INFINITY ? 0.f : mnew;
+        corr[hf] = exp2f(mx[mt][hf] - muse[hf]);
+        mx[mt][hf] = mnew;
+        ls[mt][hf] *= corr[hf];
+      }
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+#pragma unroll
+        for (int e4 = 0; e4 < 4; ++e4) {
+          const float p = exp2f(sacc[mt][j][e4] - muse[e4 >> 1]);
+          sacc[mt][j][e4] = p;
+          ls[mt][e4 >> 1] += p;
+        }
+#pragma unroll
+      for (int i = 0; i < DH / 8; ++i) {
+        oacc[mt][i][0] *= corr[0];
+        oacc[mt][i][1] *= corr[0];
+        oacc[mt][i][2] *= corr[1];
+        oacc[mt][i][3] *= corr[1];
+      }
+    }
+    // O += P V over this warp's 16 keys
+    uint32_t pa[MT][4];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+      pa[mt][0] = pack_bf16(sacc[mt][0][0], sacc[mt][0][1]);
+      pa[mt][1] = pack_bf16(sacc[mt][0][2], sacc[mt][0][3]);
+      pa[mt][2] = pack_bf16(sacc[mt][1][0], sacc[mt][1][1]);
+      pa[mt][3] = pack_bf16(sacc[mt][1][2], sacc[mt][1][3]);
+    }
+#pragma unroll
+    for (int dp = 0; dp < DH / 16; ++dp) {
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4_t(smem_u32(cV + swz<DH>(warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8, dp * 16 + (lane >> 4) * 8)),
+                b0, b1, b2, b3);
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        mma_bf16_16816(oacc[mt][2 * dp], pa[mt], b0, b1);
+        mma_bf16_16816(oacc[mt][2 * dp + 1], pa[mt], b2, b3);
+      }
+    }
+  }
+
+  // merge the 4 warps' partials in shared memory (the K/V ring is free now)
+  cp_async_wait<0>();
+  __syncthreads();
+  float* sO = reinterpret_cast<float*>(sK);  // [4][MT*16][DH]
+  float* sM = sO + 4 * MT * 16 * DH;         // [4][MT*16]
+  float* sL = sM + 4 * MT * 16;              // [4][MT*16]
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+    for (int hf = 0; hf < 2; ++hf) {
+      ls[mt][hf] += __shfl_xor_sync(0xffffffffu, ls[mt][hf], 1);
+      ls[mt][hf] += __shfl_xor_sync(0xffffffffu, ls[mt][hf], 2);
+      const int row = mt * 16 + g4 + 8 * hf;
+      if (t4 == 0) {
+        sM[warp * MT * 16 + row] = mx[mt][hf];
+        sL[warp * MT * 16 + row] = ls[mt][hf];
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < DH / 8; ++i)
+#pragma unroll
+      for (int e4 = 0; e4 < 4; ++e4) {
+        const int row = mt * 16 + g4 + 8 * (e4 >> 1), col = i * 8 + 2 * t4 + (e4 & 1);
+        sO[(warp * MT * 16 + row) * DH + col] = oacc[mt][i][e4];
+      }
+  }
+  __syncthreads();
+  for (int idx = tid; idx < MT * 16 * DH; idx += NT) {
+    const int row = idx / DH, col = idx % DH;
+    float m = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) m = fmaxf(m, sM[w * MT * 16 + row]);
+    float o = 0.f, l = 0.f;
+    if (m != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float mw = sM[w * MT * 16 + row];
+        const float f = mw == -INFINITY ? 0.f : exp2f(mw - m);
+        o += f * sO[(w * MT * 16 + row) * DH + col];
+        l += f * sL[w * MT * 16 + row];
+      }
+    }
+    po[row * DH + col] = o;
+    if (col == 0) pml[row] = make_float2(m, l);
+  }
+}
+
+// One CTA per (K/V head x row group, sequence): merges the nsplit partials of each of
+// the group's rows and writes O (bf16, round to nearest even) and the natural-log LSE.
+template <int DH>
+__global__ void __launch_bounds__(256) combine_kernel(DecodeArgs a) {
+  __shared__ float wgt[kMaxSplit][RG];  // exp2(m_c - m) / l of each split and row
+  __shared__ float lse_row[RG];
+  const int g = blockIdx.x / a.ngroups, rg = blockIdx.x % a.ngroups, b = blockIdx.y;
+  const int rows = min(RG, a.M - rg * RG);
+  const size_t pidx0 = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit;
+  const int T = a.lens[b];
+  const bool valid = T >= 1 && T <= a.maxT;
+  if (!valid && blockIdx.x == 0 && threadIdx.x == 0) set_status(a.status, HD_DEVBIT_INDEX);
+  for (int row = threadIdx.x; row < rows; row += blockDim.x) {
+    float m = -INFINITY;
+    for (int c = 0; c < a.nsplit; ++c) m = fmaxf(m, a.part_ml[(pidx0 + c) * RG + row].x);
+    float l = 0.f;
+    for (int c = 0; c < a.nsplit; ++c) {
+      const float2 ml = a.part_ml[(pidx0 + c) * RG + row];
+      const float f = (ml.x == -INFINITY || m == -INFINITY) ? 0.f : exp2f(ml.x - m);
+      wgt[c][row] = f;
+      l += f * ml.y;
+    }
+    const float inv = (valid && l > 0.f) ? 1.f / l : 0.f;
+    for (int c = 0; c < a.nsplit; ++c) wgt[c][row] *= inv;
+    lse_row[row] = (valid && l > 0.f) ? (m + __log2f(l)) * 0.6931471805599453f : -INFINITY;
+  }
+  __syncthreads();
+  constexpr int C8 = DH / 8;
+  for (int idx = threadIdx.x; idx < rows * C8; idx += blockDim.x) {
+    const int row = idx / C8, c8 = idx % C8;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int c = 0; c < a.nsplit; ++c) {
+      const float f = wgt[c][row];
+      if (f == 0.f) continue;
+      const float4* src = reinterpret_cast<const float4*>(a.part_o + ((pidx0 + c) * RG + row) * DH + c8 * 8);
+      const float4 x0 = src[0], x1 = src[1];
+      acc[0] += f * x0.x;
+      acc[1] += f * x0.y;
+      acc[2] += f * x0.z;
+      acc[3] += f * x0.w;
+      acc[4] += f * x1.x;
+      acc[5] += f * x1.y;
+      acc[6] += f * x1.z;
+      acc[7] += f * x1.w;
+    }
+    const int r = rg * RG + row, s = r / a.G, h = g * a.G + r % a.G;
+    uint4 out;
+    out.x = pack_bf16(acc[0], acc[1]);
+    out.y = pack_bf16(acc[2], acc[3]);
+    out.z = pack_bf16(acc[4], acc[5]);
+    out.w = pack_bf16(acc[6], acc[7]);
+    *reinterpret_cast<uint4*>(a.o + (((long long)b * a.n + s) * a.Hq + h) * DH + c8 * 8) = out;
+    if (c8 == 0 && a.lse != nullptr) a.lse[((long long)b * a.Hq + h) * a.n + s] = lse_row[row];
+  }
+}
+
+// The new token's n K and V rows into the cache at positions (T-1)n + s: one warp per
+// (sequence, stream), 16-byte vectors.  A length outside [1, Lcap] writes nothing and
+// sets HD_DEVBIT_INDEX.
+__global__ void __launch_bounds__(256) append_kernel(const uint4* __restrict__ kn, const uint4* __restrict__ vn,
+                                                     uint4* __restrict__ kc, uint4* __restrict__ vc,
+                                                     const int32_t* __restrict__ lens, int B, int Lcap, int n,
+                                                     int row16, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const long long w = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (w >= (long long)B * n) return;
+  const int b = (int)(w / n), s = (int)(w % n);
+  const int T = lens[b];
+  if (T < 1 || T > Lcap) {
+    if (lane == 0 && s == 0) set_status(status, HD_DEVBIT_INDEX);
+    return;
+  }
+  const long long dst = ((long long)b * Lcap * n + (long long)(T - 1) * n + s) * row16;
+  const long long src = w * row16;
+  for (int i = lane; i < row16; i += 32) {
+    kc[dst + i] = kn[src + i];
+    vc[dst + i] = vn[src + i];
+  }
+}
+}  // namespace dec
+
+// ------------------------------------------------------------------ host side
+struct DecodePlan {
+  int G, M, ngroups, nsplit, chunk;
+  size_t part_o_bytes, part_ml_bytes;
+};
+
+DecodePlan decode_plan(int B, int maxT, int n, int Hq, int Hkv, int Dh, int mode, int window) {
+  using namespace dec;
+  DecodePlan p;
+  p.G = Hq / Hkv;
+  p.M = n * p.G;
+  p.ngroups = (p.M + RG - 1) / RG;
+  const long long range = mode == SFA_LOCAL ? std::min<long long>((long long)maxT * n, (long long)window + n - 1)
+                                            : (long long)maxT * n;
+  const long long tiles = (range + KT - 1) / KT;
+  const long long ctas = (long long)B * Hkv * p.ngroups;
+  long long ns = (kTargetCtas + ctas - 1) / ctas;
+  ns = std::max(1LL, std::min(ns, std::min(tiles, (long long)kMaxSplit)));
+  const long long tiles_per = (tiles + ns - 1) / ns;
+  p.chunk = (int)(tiles_per * KT);
+  p.nsplit = (int)((tiles + tiles_per - 1) / tiles_per);
+  const size_t parts = (size_t)B * Hkv * p.ngroups * p.nsplit;
+  p.part_o_bytes = parts * RG * Dh * sizeof(float);
+  p.part_ml_bytes = parts * RG * sizeof(float2);
+  return p;
+}
+
+size_t decode_ws_bytes(const DecodePlan& p) { return ((p.part_o_bytes + 255) & ~size_t(255)) + p.part_ml_bytes; }
+
+template <int DH, int MT>
+static cudaError_t launch_decode_t(const dec::DecodeArgs& a, cudaStream_t st) {
+  using namespace dec;
+  const size_t smem = (size_t)(MT * 16 + 2 * STAGES * KT) * DH * sizeof(bf16);
+  cudaError_t e = cudaFuncSetAttribute(decode_kernel<DH, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  decode_kernel<DH, MT><<<dim3(a.nsplit, a.Hkv * a.ngroups, a.B), NT, smem, st>>>(a);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  combine_kernel<DH><<<dim3(a.Hkv * a.ngroups, a.B), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sfa_decode(const void* q, const void* kc, const void* vc, const int32_t* lens, void* o,
+                              float* lse, int B, int maxT, int Lcap, int n, int Hq, int Hkv, int Dh, float scale,
+                              int mode, int window, void* ws, int32_t* status, cudaStream_t st) {
+  const DecodePlan p = decode_plan(B, maxT, n, Hq, Hkv, Dh, mode, window);
+  dec::DecodeArgs a;
+  a.q = (const bf16*)q;
+  a.kc = (const bf16*)kc;
+  a.vc = (const bf16*)vc;
+  a.lens = lens;
+  a.o = (bf16*)o;
+  a.lse = lse;
+  a.part_o = static_cast<float*>(ws);
+  a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + ((p.part_o_bytes + 255) & ~size_t(255)));
+  a.status = status;
+  a.B = B;
+  a.Lcap = Lcap;
+  a.maxT = maxT;
+  a.n = n;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.G = p.G;
+  a.M = p.M;
+  a.ngroups = p.ngroups;
+  a.nsplit = p.nsplit;
+  a.chunk = p.chunk;
+  a.mode = mode;
+  a.window = window;
+  a.scale_log2 = scale * 1.4426950408889634f;
+  const bool two = p.M > 16;  // a row group of more than 16 rows takes two m16 tiles
+  if (Dh == 64) return two ? launch_decode_t<64, 2>(a, st) : launch_decode_t<64, 1>(a, st);
+  return two ? launch_decode_t<128, 2>(a, st) : launch_decode_t<128, 1>(a, st);
+}
+
+cudaError_t launch_kv_append(const void* kn, const void* vn, void* kc, void* vc, const int32_t* lens, int B,
+                             int Lcap, int n, int Hkv, int Dh, int32_t* status, cudaStream_t st) {
+  const long long warps = (long long)B * n;
+  dec::append_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(
+      (const uint4*)kn, (const uint4*)vn, (uint4*)kc, (uint4*)vc, lens, B, Lcap, n, Hkv * Dh / 8, status);
+  return cudaGetLastError();
+}
+
+}  // namespace hdsfa

@@ -141,3 +141,34 @@ def test_select_final_validation(lib):
         assert f(P(FAKE + 4), P(FAKE), 1, 4, 2, 16, None) == 1
         assert f(P(FAKE), None, 1, 4, 2, 16, None) == 1
         assert f(P(FAKE), P(FAKE), 1, 0, 2, 16, None) == 1
+
+
+def test_decode_workspace_and_validation(lib):
+    P, Z, F = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_float
+    need = lib.sfa_decode_workspace_bytes(1, 100, 4, 32, 8, 128, 1, 0)
+    assert need > 0
+    assert lib.sfa_decode_workspace_bytes(1, 100, 4, 32, 8, 96, 1, 0) == 0     # Dh 96
+    assert lib.sfa_decode_workspace_bytes(1, 100, 4, 32, 6, 128, 1, 0) == 0    # Hq % Hkv
+    assert lib.sfa_decode_workspace_bytes(1, 100, 4, 32, 8, 128, 2, 0) == 0    # LOCAL needs a window
+
+    def call(q=FAKE, lens=FAKE, lse=None, B=1, T=100, Lcap=100, n=4, Hq=32, Hkv=8, Dh=128, mode=1, w=0,
+             ws=FAKE, wsb=need):
+        return lib.sfa_decode(P(q), P(FAKE), P(FAKE), P(lens), P(FAKE), P(lse), B, T, Lcap, n, Hq, Hkv, Dh, F(0.0),
+                              mode, w, P(ws), Z(wsb), None, None)
+
+    assert call(q=FAKE + 2) == 1
+    assert call(lens=0) == 1 and call(lens=FAKE + 2) == 1
+    assert call(lse=FAKE + 2) == 1
+    assert call(T=101) == 1                    # max_tokens beyond the capacity
+    assert call(Hkv=6) == 1 and call(B=0) == 1 and call(mode=3) == 1
+    assert call(Dh=96) == 2
+    assert call(wsb=need - 1) == 4
+    assert call(ws=0) == 4
+
+
+def test_kv_append_validation(lib):
+    P = ctypes.c_void_p
+    assert lib.sfa_kv_append(P(FAKE), P(FAKE), P(FAKE), P(FAKE), None, 1, 10, 4, 8, 128, None, None) == 1
+    assert lib.sfa_kv_append(P(FAKE), P(FAKE + 8), P(FAKE), P(FAKE), P(FAKE), 1, 10, 4, 8, 128, None, None) == 1
+    assert lib.sfa_kv_append(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 0, 4, 8, 128, None, None) == 1
+    assert lib.sfa_kv_append(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 10, 4, 8, 12, None, None) == 1

@@ -1,0 +1,148 @@
+"""GPU parity of decoding over the expanded KV cache (Sec. 3.2 "Inference Cost") and
+of the cache append, against the oracle, through the C ABI.
+
+Tolerances as for the forward: max|dO| <= 2e-2, max|dLSE| <= 1e-3 (bf16 inputs, fp32
+accumulation, P rounded to bf16 for its MMA); the append is bit-exact."""
+import pytest
+import torch
+
+import oracle
+from paper_2607_08186_gb300 import binding, build, inputs
+
+pytestmark = pytest.mark.gpu
+
+WITHIN, CROSS, LOCAL = inputs.WITHIN, inputs.CROSS, inputs.LOCAL
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    build.build()
+
+
+def _case(B, Lcap, n, Hq, Hkv, Dh, seed):
+    q = inputs.normal_bf16((B, n, Hq, Dh), seed)
+    kc = inputs.normal_bf16((B, Lcap * n, Hkv, Dh), seed + 1)
+    vc = inputs.normal_bf16((B, Lcap * n, Hkv, Dh), seed + 2)
+    return q, kc, vc
+
+
+def _gpu_decode(q, kc, vc, lens, n, mode, window=0, max_tokens=None, status=None, reps=1):
+    B, _, Hq, Dh = q.shape
+    Lcap, Hkv = kc.shape[1] // n, kc.shape[2]
+    T = Lcap if max_tokens is None else max_tokens
+    ws = torch.empty(binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode, window), dtype=torch.uint8,
+                     device="cuda")
+    qd, kd, vd, ld = q.cuda(), kc.cuda(), vc.cuda(), lens.cuda()
+    outs = []
+    for _ in range(reps):
+        o = torch.full((B, n, Hq, Dh), 7.0, dtype=torch.bfloat16, device="cuda")
+        lse = torch.full((B, Hq, n), 7.0, dtype=torch.float32, device="cuda")
+        binding.sfa_decode(qd, kd, vd, ld, o, n, mode, ws, max_tokens=T, lse=lse, window=window,
+                           dev_status=status)
+        torch.cuda.synchronize()
+        outs.append((o.cpu(), lse.cpu()))
+    return outs if reps > 1 else outs[0]
+
+
+def _check(q, kc, vc, lens, n, mode, window=0, max_tokens=None):
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    o, lse = _gpu_decode(q, kc, vc, lens, n, mode, window, max_tokens, st)
+    o_r, lse_r, bad = oracle.decode(q, kc, vc, lens, n, mode, window=window)
+    assert bad == 0 and int(st.item()) == 0
+    eo = float((o.double() - o_r).abs().max())
+    el = float((lse.double() - lse_r).abs().max())
+    assert eo <= 2e-2 and el <= 1e-3, (eo, el)
+
+
+@pytest.mark.parametrize("mode,w", [(WITHIN, 0), (CROSS, 0), (LOCAL, 7)])
+def test_tiny(mode, w):
+    # B=2, n=2, Hq=4, Hkv=2 (8 query rows of 16), Dh=64, ragged lengths 40 and 17
+    q, kc, vc = _case(2, 40, 2, 4, 2, 64, 1)
+    _check(q, kc, vc, torch.tensor([40, 17], dtype=torch.int32), 2, mode, w)
+
+
+@pytest.mark.parametrize("mode,w", [(WITHIN, 0), (CROSS, 0), (LOCAL, 1), (LOCAL, 100)])
+@pytest.mark.parametrize("n,Hq,Hkv", [(4, 32, 8), (8, 32, 8), (8, 64, 8), (1, 8, 8), (3, 6, 2)])
+def test_shapes_ragged(mode, w, n, Hq, Hkv):
+    # query rows per K/V head: 16 (one m16 tile), 32 (two), 64 (two CTAs per head),
+    # 1 and 9; lengths 1, 129 and the full capacity in one batch
+    Lcap = 300
+    q, kc, vc = _case(3, Lcap, n, Hq, Hkv, 128, n + Hq)
+    _check(q, kc, vc, torch.tensor([Lcap, 1, 129], dtype=torch.int32), n, mode, w)
+
+
+def test_max_tokens_below_capacity():
+    q, kc, vc = _case(2, 500, 4, 8, 2, 128, 5)
+    _check(q, kc, vc, torch.tensor([200, 77], dtype=torch.int32), 4, CROSS, max_tokens=200)
+
+
+def test_bad_lengths_zero_rows_and_flag():
+    q, kc, vc = _case(3, 50, 2, 4, 2, 128, 6)
+    lens = torch.tensor([0, 50, 51], dtype=torch.int32)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    o, lse = _gpu_decode(q, kc, vc, lens, 2, CROSS, status=st)
+    assert int(st.item()) & binding.HD_DEVBIT_INDEX
+    o_r, lse_r, bad = oracle.decode(q, kc, vc, lens, 2, CROSS)
+    assert bad == 2
+    assert torch.count_nonzero(o[0]) == 0 and torch.count_nonzero(o[2]) == 0
+    assert torch.isinf(lse[0]).all() and torch.isinf(lse[2]).all()
+    assert float((o[1].double() - o_r[1]).abs().max()) <= 2e-2
+
+
+def test_deterministic():
+    q, kc, vc = _case(2, 700, 4, 32, 8, 128, 7)
+    runs = _gpu_decode(q, kc, vc, torch.tensor([700, 350], dtype=torch.int32), 4, CROSS, reps=3)
+    for o, lse in runs[1:]:
+        assert torch.equal(o.view(torch.int16), runs[0][0].view(torch.int16))
+        assert torch.equal(lse, runs[0][1])
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_full_size(mode):
+    # Qwen3-8B-class heads, n = 4, an 8192-token context (32768 cached positions), B = 2
+    # with one shorter sequence; every output row checked against the oracle
+    q, kc, vc = _case(2, 8192, 4, 32, 8, 128, 8)
+    _check(q, kc, vc, torch.tensor([8192, 5000], dtype=torch.int32), 4, mode)
+
+
+def test_kv_append_bit_exact_and_flag():
+    B, n, Lcap, Hkv, Dh = 4, 4, 33, 8, 128
+    kc = inputs.normal_bf16((B, Lcap * n, Hkv, Dh), 9)
+    vc = inputs.normal_bf16((B, Lcap * n, Hkv, Dh), 10)
+    kn = inputs.normal_bf16((B, n, Hkv, Dh), 11)
+    vn = inputs.normal_bf16((B, n, Hkv, Dh), 12)
+    lens = torch.tensor([1, 33, 17, 34], dtype=torch.int32)        # the last is out of range
+    kd, vd = kc.cuda(), vc.cuda()
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    binding.sfa_kv_append(kn.cuda(), vn.cuda(), kd, vd, lens.cuda(), n, dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & binding.HD_DEVBIT_INDEX
+    k_ref, bad = oracle.kv_append(kn, kc, lens, n)
+    v_ref, _ = oracle.kv_append(vn, vc, lens, n)
+    assert bad == 1
+    assert torch.equal(kd.cpu().view(torch.int16), k_ref.view(torch.int16))
+    assert torch.equal(vd.cpu().view(torch.int16), v_ref.view(torch.int16))
+
+
+def test_append_then_decode_equals_forward_rows():
+    # a prefilled cache (the forward's K/V) plus one appended token decodes to the
+    # forward's rows of that token, for every mask
+    B, L, n, Hq, Hkv, Dh = 1, 50, 4, 8, 2, 128
+    q, k, v = inputs.attn_inputs(inputs.AttnShape(B, L, n, Hq, Hkv, Dh), seed=13, with_grad=False)
+    kd = torch.zeros(B, L * n, Hkv, Dh, dtype=torch.bfloat16, device="cuda")
+    vd = torch.zeros_like(kd)
+    kd[:, :(L - 1) * n] = k[:, :(L - 1) * n].cuda()
+    vd[:, :(L - 1) * n] = v[:, :(L - 1) * n].cuda()
+    lens = torch.tensor([L], dtype=torch.int32)
+    binding.sfa_kv_append(k[:, (L - 1) * n:].contiguous().cuda(), v[:, (L - 1) * n:].contiguous().cuda(), kd, vd,
+                          lens.cuda(), n)
+    torch.cuda.synchronize()
+    qn = q[:, (L - 1) * n:].contiguous()
+    for mode, w in ((WITHIN, 0), (CROSS, 0), (LOCAL, 9)):
+        o, lse = _gpu_decode(qn, kd.cpu(), vd.cpu(), lens, n, mode, w)
+        rows = [(0, h, p) for h in range(Hq) for p in range((L - 1) * n, L * n)]
+        o_r, lse_r = oracle.sfa_fwd_rows(q, k, v, n, mode, rows, window=w)
+        got = torch.stack([o[0, p - (L - 1) * n, h] for (_, h, p) in rows]).double()
+        assert float((got - o_r).abs().max()) <= 2e-2
+        got_l = torch.tensor([float(lse[0, h, p - (L - 1) * n]) for (_, h, p) in rows], dtype=torch.float64)
+        assert float((got_l - lse_r).abs().max()) <= 1e-3
