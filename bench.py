@@ -12,8 +12,9 @@ pair and query head) per second of the whole step, in TFLOP/s.
 The same JSON line also carries: the dominant kernel's roofline, the end-to-end
 number through the C ABI with host buffers, the CPU oracle baseline, and under
 "extras" the CROSS (full cross-stream) layer of the same shape, the expansion-factor
-sweep, the LOCAL (sliding-window) layer at windows of 1024 and 4096 positions, and
-the HBM bandwidth of the expansion backward and the final-stream selection.
+sweep, the LOCAL (sliding-window) layer at windows of 1024 and 4096 positions, the
+HBM bandwidth of the expansion backward and the final-stream selection, and of the
+decoding step over the expanded KV cache.
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the paper publishes no implementation to run).
@@ -368,6 +369,46 @@ def measure_expansion_backward(dev, hbm_peak: float, V: int = GATHER_V):
     return out
 
 
+def measure_decode(dev, hbm_peak: float, quick: bool = False):
+    """Decoding step (Sec. 3.2) with Qwen3-8B-class heads (Hq=32, Hkv=8, Dh=128), n=4:
+    the new token's 4 positions against a context of T tokens (4T cached positions) for
+    batch B, WITHIN and CROSS layers.  Algorithmic bytes: the visible cached K and V rows
+    (B*T*n*Hkv*Dh*2 bytes each) plus q and o; rotating cache sets keep every call out of L2."""
+    from paper_2607_08186_gb300 import binding
+    n, Hq, Hkv, Dh = 4, 32, 8, 128
+    grid = [(1, 8192), (4, 8192), (16, 8192), (1, 32768), (16, 32768)]
+    if quick:
+        grid = [(1, 8192), (16, 8192)]
+    out = []
+    g = torch.Generator(device=dev)
+    g.manual_seed(41)
+    for B, T in grid:
+        cache_bytes = 2 * B * T * n * Hkv * Dh * 2
+        S = max(1, min(3, -(-400_000_000 // cache_bytes)))
+        sets = []
+        for _ in range(S):
+            kc = torch.randn(B, T * n, Hkv, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+            vc = torch.randn(B, T * n, Hkv, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+            q = torch.randn(B, n, Hq, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+            sets.append((q, kc, vc))
+        lens = torch.full((B,), T, dtype=torch.int32, device=dev)
+        o = torch.empty(B, n, Hq, Dh, dtype=torch.bfloat16, device=dev)
+        lse = torch.empty(B, Hq, n, dtype=torch.float32, device=dev)
+        row = {"B": B, "context_tokens": T, "cached_positions": T * n}
+        for mode in (WITHIN, CROSS):
+            ws = torch.empty(binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
+                             device=dev)
+            t = time_op(lambda k: binding.sfa_decode(sets[k][0], sets[k][1], sets[k][2], lens, o, n, mode, ws,
+                                                     max_tokens=T, lse=lse), S)
+            nbytes = cache_bytes + 2 * B * n * Hq * Dh * 2
+            row[MODE_NAME[mode]] = {"us": t * 1e6, "gbs": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / hbm_peak}
+        out.append(row)
+        del sets, o, lse
+        torch.cuda.empty_cache()
+    return {"workload": "decode step, Hq=32 Hkv=8 Dh=128 n=4, all sequences at the context length; "
+                        "bytes = cached K+V rows read + q + o", "rows": out}
+
+
 # ---------------------------------------------------------------- ncu traffic record
 # ABI phase -> (kernel symbol, source file) of the implementation the library runs.
 KERNEL_OF = {
@@ -475,6 +516,8 @@ def main():
     ap.add_argument("--no-extras", action="store_true", help="skip the extras (CROSS / LOCAL layers, n sweep, expansion backward) and the CPU baseline")
     ap.add_argument("--expand-bwd-only", action="store_true",
                     help="time only the expansion backward and final-stream selection (JSON line)")
+    ap.add_argument("--decode-only", action="store_true",
+                    help="time only the decoding step over the serving grid (JSON line)")
     ap.add_argument("--vocab", type=int, default=GATHER_V,
                     help="table rows V for --expand-bwd-only (smaller V for traffic captures)")
     ap.add_argument("--layer-only", choices=["within", "cross", "local"], default=None,
@@ -496,6 +539,11 @@ def main():
     barrier(ws)
     s = SHAPES[WORKLOAD]
     pk = peaks()
+    if args.decode_only:
+        r = measure_decode(dev, pk["hbm"])
+        if rank == 0:
+            print(json.dumps(r), flush=True)
+        return
     if args.expand_bwd_only:
         r = measure_expansion_backward(dev, pk["hbm"], V=args.vocab)
         if rank == 0:
@@ -609,6 +657,7 @@ def main():
                         "bwd_main_tflops": attn_flops(s, LOCAL, BWD_FLOP, w) / r["bwd_main_s"] / 1e12})
         extras["local_layer"] = {"workload": f"{WORKLOAD}_local", "windows": loc}
         extras["expansion_backward"] = measure_expansion_backward(dev, pk["hbm"])
+        extras["decode"] = measure_decode(dev, pk["hbm"], quick=True)
         out["extras"] = extras
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:

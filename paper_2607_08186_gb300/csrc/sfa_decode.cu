@@ -37,7 +37,6 @@ constexpr int KT = 64;       // cached positions per pipeline stage
 constexpr int STAGES = 3;
 constexpr int RG = 32;       // query rows per CTA at most (two m16 tiles)
 constexpr int kMaxSplit = 128;
-constexpr int kTargetCtas = 152 * 4;
 
 struct DecodeArgs {
   const bf16* q;        // [B][n][Hq][Dh]
@@ -121,6 +120,14 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
       rs_[mt][hf] = r < a.M ? r / a.G : -1;
       rq[mt][hf] = (T - 1) * a.n + (r < a.M ? r / a.G : 0);
     }
+  // stream of this thread's keys: when n divides 16 and k0, every warp's first key is a
+  // multiple of n, so the stream of key kb + j*8 + 2*t4 + e is fixed per thread
+  const bool kst_fixed = (16 % a.n) == 0 && (k0 % a.n) == 0;
+  int kst0[2][2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j)
+#pragma unroll
+    for (int e = 0; e < 2; ++e) kst0[j][e] = (j * 8 + 2 * t4 + e) % a.n;
   float mx[MT][2], ls[MT][2], oacc[MT][DH / 8][4];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
@@ -165,7 +172,7 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         kp[j][e] = kb + j * 8 + 2 * t4 + e;
-        kst[j][e] = a.mode == SFA_WITHIN ? kp[j][e] % a.n : 0;
+        kst[j][e] = a.mode != SFA_WITHIN ? 0 : (kst_fixed ? kst0[j][e] : kp[j][e] % a.n);
       }
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
@@ -278,59 +285,61 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
   }
 }
 
-// One CTA per (K/V head x row group, sequence): merges the nsplit partials of each of
-// the group's rows and writes O (bf16, round to nearest even) and the natural-log LSE.
+// CTA (K/V head x row group, sequence, 8-column slice); one warp per query row, its
+// lanes over the splits: the row's max and sum by warp reductions, then the slice of
+// O as the weighted sum of the splits' partial slices, written as bf16 (round to
+// nearest even); the first slice's CTA also writes the natural-log LSE.
 template <int DH>
 __global__ void __launch_bounds__(256) combine_kernel(DecodeArgs a) {
-  __shared__ float wgt[kMaxSplit][RG];  // exp2(m_c - m) / l of each split and row
-  __shared__ float lse_row[RG];
-  const int g = blockIdx.x / a.ngroups, rg = blockIdx.x % a.ngroups, b = blockIdx.y;
+  const int g = blockIdx.x / a.ngroups, rg = blockIdx.x % a.ngroups, b = blockIdx.y, c8 = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rows = min(RG, a.M - rg * RG);
   const size_t pidx0 = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit;
   const int T = a.lens[b];
   const bool valid = T >= 1 && T <= a.maxT;
-  if (!valid && blockIdx.x == 0 && threadIdx.x == 0) set_status(a.status, HD_DEVBIT_INDEX);
-  for (int row = threadIdx.x; row < rows; row += blockDim.x) {
+  if (!valid && blockIdx.x == 0 && c8 == 0 && threadIdx.x == 0) set_status(a.status, HD_DEVBIT_INDEX);
+  for (int row = warp; row < rows; row += 8) {
     float m = -INFINITY;
-    for (int c = 0; c < a.nsplit; ++c) m = fmaxf(m, a.part_ml[(pidx0 + c) * RG + row].x);
-    float l = 0.f;
-    for (int c = 0; c < a.nsplit; ++c) {
+    for (int c = lane; c < a.nsplit; c += 32) m = fmaxf(m, a.part_ml[(pidx0 + c) * RG + row].x);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+    float l = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int c = lane; c < a.nsplit; c += 32) {
       const float2 ml = a.part_ml[(pidx0 + c) * RG + row];
       const float f = (ml.x == -INFINITY || m == -INFINITY) ? 0.f : exp2f(ml.x - m);
-      wgt[c][row] = f;
       l += f * ml.y;
+      if (f != 0.f) {
+        const float4* src = reinterpret_cast<const float4*>(a.part_o + ((pidx0 + c) * RG + row) * DH + c8 * 8);
+        const float4 x0 = src[0], x1 = src[1];
+        acc[0] += f * x0.x;
+        acc[1] += f * x0.y;
+        acc[2] += f * x0.z;
+        acc[3] += f * x0.w;
+        acc[4] += f * x1.x;
+        acc[5] += f * x1.y;
+        acc[6] += f * x1.z;
+        acc[7] += f * x1.w;
+      }
     }
-    const float inv = (valid && l > 0.f) ? 1.f / l : 0.f;
-    for (int c = 0; c < a.nsplit; ++c) wgt[c][row] *= inv;
-    lse_row[row] = (valid && l > 0.f) ? (m + __log2f(l)) * 0.6931471805599453f : -INFINITY;
-  }
-  __syncthreads();
-  constexpr int C8 = DH / 8;
-  for (int idx = threadIdx.x; idx < rows * C8; idx += blockDim.x) {
-    const int row = idx / C8, c8 = idx % C8;
-    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    for (int c = 0; c < a.nsplit; ++c) {
-      const float f = wgt[c][row];
-      if (f == 0.f) continue;
-      const float4* src = reinterpret_cast<const float4*>(a.part_o + ((pidx0 + c) * RG + row) * DH + c8 * 8);
-      const float4 x0 = src[0], x1 = src[1];
-      acc[0] += f * x0.x;
-      acc[1] += f * x0.y;
-      acc[2] += f * x0.z;
-      acc[3] += f * x0.w;
-      acc[4] += f * x1.x;
-      acc[5] += f * x1.y;
-      acc[6] += f * x1.z;
-      acc[7] += f * x1.w;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+      l += __shfl_xor_sync(0xffffffffu, l, off);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], off);
     }
-    const int r = rg * RG + row, s = r / a.G, h = g * a.G + r % a.G;
-    uint4 out;
-    out.x = pack_bf16(acc[0], acc[1]);
-    out.y = pack_bf16(acc[2], acc[3]);
-    out.z = pack_bf16(acc[4], acc[5]);
-    out.w = pack_bf16(acc[6], acc[7]);
-    *reinterpret_cast<uint4*>(a.o + (((long long)b * a.n + s) * a.Hq + h) * DH + c8 * 8) = out;
-    if (c8 == 0 && a.lse != nullptr) a.lse[((long long)b * a.Hq + h) * a.n + s] = lse_row[row];
+    if (lane == 0) {
+      const bool ok = valid && l > 0.f;
+      const float inv = ok ? 1.f / l : 0.f;
+      const int r = rg * RG + row, s = r / a.G, h = g * a.G + r % a.G;
+      uint4 out;
+      out.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      out.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      out.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+      out.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+      *reinterpret_cast<uint4*>(a.o + (((long long)b * a.n + s) * a.Hq + h) * DH + c8 * 8) = out;
+      if (c8 == 0 && a.lse != nullptr)
+        a.lse[((long long)b * a.Hq + h) * a.n + s] = ok ? (m + __log2f(l)) * 0.6931471805599453f : -INFINITY;
+    }
   }
 }
 
@@ -375,9 +384,20 @@ DecodePlan decode_plan(int B, int maxT, int n, int Hq, int Hkv, int Dh, int mode
                                             : (long long)maxT * n;
   const long long tiles = (range + KT - 1) / KT;
   const long long ctas = (long long)B * Hkv * p.ngroups;
-  long long ns = (kTargetCtas + ctas - 1) / ctas;
-  ns = std::max(1LL, std::min(ns, std::min(tiles, (long long)kMaxSplit)));
-  const long long tiles_per = (tiles + ns - 1) / ns;
+  // resident decode CTAs: two per SM at head dim 128 (104 KB of shared memory), four at 64
+  const long long resident = 152LL * (Dh == 64 ? 4 : 2);
+  // split count: least (waves x (tiles per CTA + a fixed cost of about two tiles))
+  long long best = 1, best_cost = -1;
+  for (long long ns = 1; ns <= std::min(tiles, (long long)kMaxSplit); ++ns) {
+    const long long per = (tiles + ns - 1) / ns, used = (tiles + per - 1) / per;
+    if (used != ns) continue;  // another ns gives the same chunks
+    const long long cost = ((ctas * ns + resident - 1) / resident) * (per + 2);
+    if (best_cost < 0 || cost < best_cost) {
+      best = ns;
+      best_cost = cost;
+    }
+  }
+  const long long tiles_per = (tiles + best - 1) / best;
   p.chunk = (int)(tiles_per * KT);
   p.nsplit = (int)((tiles + tiles_per - 1) / tiles_per);
   const size_t parts = (size_t)B * Hkv * p.ngroups * p.nsplit;
@@ -397,7 +417,7 @@ static cudaError_t launch_decode_t(const dec::DecodeArgs& a, cudaStream_t st) {
   decode_kernel<DH, MT><<<dim3(a.nsplit, a.Hkv * a.ngroups, a.B), NT, smem, st>>>(a);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  combine_kernel<DH><<<dim3(a.Hkv * a.ngroups, a.B), 256, 0, st>>>(a);
+  combine_kernel<DH><<<dim3(a.Hkv * a.ngroups, a.B, DH / 8), 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 
