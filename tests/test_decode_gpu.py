@@ -146,3 +146,64 @@ def test_append_then_decode_equals_forward_rows():
         assert float((got - o_r).abs().max()) <= 2e-2
         got_l = torch.tensor([float(lse[0, h, p - (L - 1) * n]) for (_, h, p) in rows], dtype=torch.float64)
         assert float((got_l - lse_r).abs().max()) <= 1e-3
+
+
+def test_serving_loop_in_a_cuda_graph():
+    # one step of a serving loop (append the new token's n K/V rows, then an intra-stream
+    # and a cross-stream decode over the cache) captured once as a CUDA graph and replayed
+    # while the sequences grow; every replay equals the oracle on the cache as it stands
+    B, n, Hq, Hkv, Dh, Lcap = 2, 4, 8, 2, 128, 64
+    lens0 = [20, 33]
+    kc = torch.zeros(B, Lcap * n, Hkv, Dh, dtype=torch.bfloat16, device="cuda")
+    vc = torch.zeros_like(kc)
+    for b, t in enumerate(lens0):
+        kc[b, :t * n] = inputs.normal_bf16((t * n, Hkv, Dh), 20 + b).cuda()
+        vc[b, :t * n] = inputs.normal_bf16((t * n, Hkv, Dh), 30 + b).cuda()
+    lens = torch.tensor(lens0, dtype=torch.int32, device="cuda")
+    qs = torch.zeros(B, n, Hq, Dh, dtype=torch.bfloat16, device="cuda")
+    kn, vn = torch.zeros(B, n, Hkv, Dh, dtype=torch.bfloat16, device="cuda"), torch.zeros(B, n, Hkv, Dh,
+                                                                                          dtype=torch.bfloat16,
+                                                                                          device="cuda")
+    outs = {m: (torch.empty(B, n, Hq, Dh, dtype=torch.bfloat16, device="cuda"),
+                torch.empty(B, Hq, n, dtype=torch.float32, device="cuda")) for m in (WITHIN, CROSS)}
+    wss = {m: torch.empty(binding.sfa_decode_workspace_bytes(B, Lcap, n, Hq, Hkv, Dh, m), dtype=torch.uint8,
+                          device="cuda") for m in (WITHIN, CROSS)}
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+
+    def step():
+        binding.sfa_kv_append(kn, vn, kc, vc, lens, n, dev_status=st)
+        for m in (WITHIN, CROSS):
+            binding.sfa_decode(qs, kc, vc, lens, outs[m][0], n, m, wss[m], max_tokens=Lcap, lse=outs[m][1],
+                               dev_status=st)
+
+    lens += 1
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()  # warm-up outside the capture (also the first step of the loop)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    for it in range(3):
+        if it > 0:  # the captured step reads these buffers: refill them, grow the sequences
+            lens += 1
+            qs.copy_(inputs.normal_bf16((B, n, Hq, Dh), 100 + it).cuda())
+            kn.copy_(inputs.normal_bf16((B, n, Hkv, Dh), 200 + it).cuda())
+            vn.copy_(inputs.normal_bf16((B, n, Hkv, Dh), 300 + it).cuda())
+            graph.replay()
+        else:  # the warm-up already ran step 0 on zero q / K / V rows: run it again with data
+            qs.copy_(inputs.normal_bf16((B, n, Hq, Dh), 100).cuda())
+            kn.copy_(inputs.normal_bf16((B, n, Hkv, Dh), 200).cuda())
+            vn.copy_(inputs.normal_bf16((B, n, Hkv, Dh), 300).cuda())
+            graph.replay()
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0
+        lh = lens.cpu()
+        for m in (WITHIN, CROSS):
+            o_r, lse_r, bad = oracle.decode(qs.cpu(), kc.cpu(), vc.cpu(), lh, n, m)
+            assert bad == 0
+            assert float((outs[m][0].cpu().double() - o_r).abs().max()) <= 2e-2
+            assert float((outs[m][1].cpu().double() - lse_r).abs().max()) <= 1e-3
+    assert lens.cpu().tolist() == [t + 3 for t in lens0]
