@@ -237,6 +237,38 @@ def sfa_fwd_rows(q, k, v, n, mode, rows, scale=None, window=0):
     return torch.from_numpy(o), torch.from_numpy(lse)
 
 
+def _final_full(x, n):
+    """[B][L][H][Dh] -> [B][nL][H][Dh] fp64 with x at the final-stream rows t*n + n-1, zero elsewhere."""
+    xa = _f64(x)
+    B, L, H, Dh = xa.shape
+    full = np.zeros((B, n * L, H, Dh))
+    full[:, n - 1::n] = xa
+    return full
+
+
+def sfa_fwd_final(q, k, v, n: int, mode: int, scale: float | None = None, window: int = 0):
+    """Final-stream queries (the rows the loss reads, Eq. 2; the final-stream-only layers of
+    Sec. 3.1): q [B][L][Hq][Dh] are the queries of positions t*n + n-1, attending to k / v
+    [B][nL][Hkv][Dh] under the layer's mask.  By definition these are the forward's rows
+    t*n + n-1.  Returns (O fp64 [B][L][Hq][Dh], LSE fp64 [B][Hq][L])."""
+    qf = _final_full(q, n)
+    B, nL, Hq, Dh = qf.shape
+    L = nL // n
+    rows = np.array([(b, h, t * n + n - 1) for b in range(B) for h in range(Hq) for t in range(L)], dtype=np.int64)
+    o_rows, lse_rows = sfa_fwd_rows(qf, k, v, n, mode, rows, scale, window)
+    o = o_rows.numpy().reshape(B, Hq, L, Dh).transpose(0, 2, 1, 3)
+    return torch.from_numpy(np.ascontiguousarray(o)), lse_rows.reshape(B, Hq, L)
+
+
+def sfa_bwd_final(q, k, v, dout, n: int, mode: int, scale: float | None = None, window: int = 0):
+    """Gradients of the final-stream problem: the full backward with the queries and output
+    gradients of every other position set to zero (a row with zero dO adds nothing to any
+    gradient, and rows are independent).  Returns (dQ fp64 [B][L][Hq][Dh], dK, dV fp64
+    [B][nL][Hkv][Dh])."""
+    dq, dk, dv = sfa_bwd(_final_full(q, n), k, v, _final_full(dout, n), n, mode, scale, window)
+    return dq[:, n - 1::n].contiguous(), dk, dv
+
+
 def sfa_bwd(q, k, v, dout, n, mode, scale=None, window=0):
     """Full backward (reduced Jacobian form).  Returns (dQ, dK, dV) fp64."""
     qa, ka, va, da = _f64(q), _f64(k), _f64(v), _f64(dout)

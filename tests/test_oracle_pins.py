@@ -521,3 +521,59 @@ def test_kv_append_matches_indexing():
         i = int(lens[b])
         ref[b, (i - 1) * n:i * n] = new[b]
     assert torch.equal(got.view(torch.int16), ref.view(torch.int16))
+
+
+# ------------------------------------------------------------------ final-stream problems (Eq. 2, Sec. 3.1)
+def _final_mask(L, n, mode, w=0):
+    """[L][nL] boolean: final-stream query t (position t*n + n-1) sees key p'."""
+    pq = torch.arange(L)[:, None] * n + n - 1
+    pk = torch.arange(n * L)[None, :]
+    m = pk <= pq
+    if mode == oracle.WITHIN:
+        m &= (pk % n) == (n - 1)
+    if mode == oracle.LOCAL:
+        m &= (pq - pk) < w
+    return m
+
+
+@pytest.mark.parametrize("n", [1, 2, 4])
+@pytest.mark.parametrize("mode,w", [(oracle.WITHIN, 0), (oracle.CROSS, 0), (oracle.LOCAL, 6)])
+def test_final_stream_is_masked_sdpa_with_gradients(n, mode, w):
+    # torch fp64 SDPA of the L final-stream queries against the nL keys under an explicit
+    # boolean mask, and its autograd gradients
+    B, L, Hq, Hkv, Dh, scale = 2, 9, 4, 2, 8, 0.45
+    q = _rand((B, L, Hq, Dh), 60).requires_grad_()
+    k = _rand((B, n * L, Hkv, Dh), 61).requires_grad_()
+    v = _rand((B, n * L, Hkv, Dh), 62).requires_grad_()
+    do = _rand((B, L, Hq, Dh), 63)
+    mask = _final_mask(L, n, mode, w)
+    qh = q.permute(0, 2, 1, 3)
+    kh = k.permute(0, 2, 1, 3).repeat_interleave(Hq // Hkv, dim=1)
+    vh = v.permute(0, 2, 1, 3).repeat_interleave(Hq // Hkv, dim=1)
+    ref = F.scaled_dot_product_attention(qh, kh, vh, attn_mask=mask, scale=scale).permute(0, 2, 1, 3)
+    ref.backward(do)
+    z = torch.einsum("bhqd,bhkd->bhqk", qh, kh).detach() * scale
+    lse_ref = torch.logsumexp(z.masked_fill(~mask, -math.inf), dim=-1)
+    o, lse = oracle.sfa_fwd_final(q.detach(), k.detach(), v.detach(), n, mode, scale, window=w)
+    torch.testing.assert_close(o, ref.detach(), rtol=1e-12, atol=1e-12)
+    torch.testing.assert_close(lse, lse_ref, rtol=1e-12, atol=1e-12)
+    dq, dk, dv = oracle.sfa_bwd_final(q.detach(), k.detach(), v.detach(), do, n, mode, scale, window=w)
+    torch.testing.assert_close(dq, q.grad, rtol=1e-10, atol=1e-12)
+    torch.testing.assert_close(dk, k.grad, rtol=1e-10, atol=1e-12)
+    torch.testing.assert_close(dv, v.grad, rtol=1e-10, atol=1e-12)
+
+
+def test_final_stream_within_reads_only_the_last_stream():
+    # intra-stream layer: perturbing keys/values of streams 0..n-2 changes nothing
+    B, L, n, H, Dh = 1, 6, 3, 2, 8
+    q, k, v = _rand((B, L, H, Dh), 64), _rand((B, n * L, H, Dh), 65), _rand((B, n * L, H, Dh), 66)
+    o1, _ = oracle.sfa_fwd_final(q, k, v, n, oracle.WITHIN)
+    k2, v2 = k.clone(), v.clone()
+    for s in range(n - 1):
+        k2[:, s::n] += 3.0
+        v2[:, s::n] -= 2.0
+    o2, _ = oracle.sfa_fwd_final(q, k2, v2, n, oracle.WITHIN)
+    torch.testing.assert_close(o1, o2, rtol=0, atol=0)
+    _, dk, dv = oracle.sfa_bwd_final(q, k, v, _rand((B, L, H, Dh), 67), n, oracle.WITHIN)
+    for s in range(n - 1):
+        assert torch.count_nonzero(dk[:, s::n]) == 0 and torch.count_nonzero(dv[:, s::n]) == 0
