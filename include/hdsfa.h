@@ -177,6 +177,34 @@ hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int
                              size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * sfa_fwd_final / sfa_bwd_final -- attention of the final-stream queries only (the
+ * positions t*n + n-1 the loss reads, Eq. 2) against the layer's keys over all nL
+ * positions: the layers that run only the final stream while the other streams' K/V
+ * stay as context (Sec. 3.1, KV-mirror layers).  The mask is the layer's own (Eq. 4,
+ * Fig. 2): the query of token t at position p = t*n + n-1 sees key p' iff
+ *   WITHIN  p' <= p and p' = n-1 (mod n)   (only stream n-1's keys)
+ *   CROSS   p' <= p
+ *   LOCAL   p - window < p' <= p
+ * which equals rows t*n + n-1 of sfa_fwd over the full sequence.
+ *   q, o, dout, dq : bf16 [B][L][Hq][Dh]  (dense: only the final-stream rows)
+ *   k, v, dk, dv   : bf16 [B][n*L][Hkv][Dh]
+ *   lse            : float32 [B][Hq][L], natural log (written by sfa_fwd_final)
+ * dk, dv are fully overwritten (zero for keys no final-stream query sees).
+ * workspace: >= sfa_bwd_final_workspace_bytes(...) bytes, 256-byte aligned.
+ * sfa_fwd_final takes Dh in {64, 128}; sfa_bwd_final Dh = 128 (HD_ERR_UNSUPPORTED
+ * otherwise); both run on the tcgen05 kernels (HDSFA_KERNELS=mma: HD_ERR_UNSUPPORTED).
+ */
+hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
+                          int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
+                          int32_t* dev_status, cudaStream_t stream);
+size_t sfa_bwd_final_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode);
+hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                          const void* dout, void* dq, void* dk, void* dv, int B, int L, int n, int Hq,
+                          int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
+                          void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                          cudaStream_t stream);
+
+/*
  * sfa_decode -- one decoding step over the expanded KV cache (Sec. 3.2 "Inference
  * Cost"; masks of Eq. 4 and Fig. 2).  Generation runs each new token's n streams
  * together: with T = lens[b] tokens in sequence b's cache (the new token included,

@@ -55,6 +55,12 @@ def lib():
             L.hd_select_final_stream.argtypes = [P, P, I, I, I, I, P]
             L.hd_select_final_stream_bwd.restype = I
             L.hd_select_final_stream_bwd.argtypes = [P, P, I, I, I, I, P]
+            L.sfa_fwd_final.restype = I
+            L.sfa_fwd_final.argtypes = [P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, P]
+            L.sfa_bwd_final_workspace_bytes.restype = Z
+            L.sfa_bwd_final_workspace_bytes.argtypes = [I, I, I, I, I, I, I]
+            L.sfa_bwd_final.restype = I
+            L.sfa_bwd_final.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
             L.sfa_decode_workspace_bytes.restype = Z
             L.sfa_decode_workspace_bytes.argtypes = [I, I, I, I, I, I, I, I]
             L.sfa_decode.restype = I
@@ -197,6 +203,36 @@ def sfa_bwd(q, k, v, o, lse, dout, dq, dk, dv, n, mode, workspace, softmax_scale
                          B, L, n, Hq, Hkv, Dh, float(softmax_scale), int(mode), int(window),
                          _p(workspace), _wsb(workspace),
                          _p(dev_status), _stream(stream)), "sfa_bwd")
+    return dq, dk, dv
+
+
+def _final_dims(q, k):
+    B, L, Hq, Dh = q.shape
+    if k.shape[1] % L:
+        raise ValueError("k.shape[1] must be n * L")
+    return B, L, k.shape[1] // L, Hq, k.shape[2], Dh
+
+
+def sfa_fwd_final(q, k, v, o, lse, mode, softmax_scale=0.0, window=0, dev_status=None, stream=None):
+    """Final-stream queries only (Eq. 2 rows; Sec. 3.1 final-stream-only layers): q, o [B][L][Hq][Dh],
+    k, v [B][n*L][Hkv][Dh] bf16, lse [B][Hq][L] float32."""
+    B, L, n, Hq, Hkv, Dh = _final_dims(q, k)
+    _check(lib().sfa_fwd_final(_p(q), _p(k), _p(v), _p(o), _p(lse), B, L, n, Hq, Hkv, Dh, float(softmax_scale),
+                               int(mode), int(window), _p(dev_status), _stream(stream)), "sfa_fwd_final")
+    return o, lse
+
+
+def sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode) -> int:
+    return int(lib().sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, int(mode)))
+
+
+def sfa_bwd_final(q, k, v, o, lse, dout, dq, dk, dv, mode, workspace, softmax_scale=0.0, window=0,
+                  dev_status=None, stream=None):
+    """Backward of sfa_fwd_final: dq [B][L][Hq][Dh], dk, dv [B][n*L][Hkv][Dh] (overwritten)."""
+    B, L, n, Hq, Hkv, Dh = _final_dims(q, k)
+    _check(lib().sfa_bwd_final(_p(q), _p(k), _p(v), _p(o), _p(lse), _p(dout), _p(dq), _p(dk), _p(dv), B, L, n, Hq,
+                               Hkv, Dh, float(softmax_scale), int(mode), int(window), _p(workspace),
+                               _wsb(workspace), _p(dev_status), _stream(stream)), "sfa_bwd_final")
     return dq, dk, dv
 
 

@@ -14,13 +14,38 @@
 //           its own earlier positions, which are exactly every n-th row).
 //   CROSS : one problem, Lv = nL, rs = 1, s = 0       (Fig. 2a: causal over nL).
 //   LOCAL : as CROSS plus the window lower bound       (Fig. 2b).
+//
+// Query side.  In the modes above the queries are the same virtual rows as the keys.
+// A final-stream problem (the loss rows of Eq. 2 / the final-stream-only layers of
+// Sec. 3.1) has only the L final-stream queries, in their own dense [B][L] tensors,
+// against the keys above: query row r stands at key row r*qstep + qoff of its
+// problem (CROSS / LOCAL over nL: qstep = n, qoff = n-1; WITHIN: the problem of
+// stream n-1 alone, qstep = 1, qoff = 0, kv_s0 = n-1).
 struct SfaGeom {
   int B, nL, Hq, Hkv, n;
-  int Lv;       // rows of each virtual problem
+  int Lv;       // key rows of each virtual problem
   int ns;       // problems per (b, head): n for WITHIN, 1 otherwise
   int rs;       // expanded-position step between consecutive virtual rows
   int window;   // > 0 only for LOCAL: key r' visible iff r - window < r' <= r
+  int Lq;       // query rows of each problem (= Lv when queries are the key rows)
+  int qstep, qoff;         // query row r sits at key row r*qstep + qoff (1, 0)
+  int q_nL, q_ns, q_rs;    // rows per batch, problems, row step of the query tensors (nL, ns, rs)
+  int kv_s0;               // stream of the first key problem (0)
 };
+
+// Geometry of the query-side tensors (Q, O, dO, dQ, LSE, row terms) of a problem.
+__host__ __device__ inline SfaGeom query_geom(const SfaGeom& g) {
+  SfaGeom q = g;
+  q.nL = g.q_nL;
+  q.ns = g.q_ns;
+  q.rs = g.q_rs;
+  q.Lv = g.Lq;
+  q.Lq = g.Lq;
+  q.qstep = 1;
+  q.qoff = 0;
+  q.kv_s0 = 0;
+  return q;
+}
 
 // Stream-major backward row terms (-lse*log2e, -delta) are padded per (b, h, stream)
 // to a multiple of the largest query tile any backward kernel reads at once.

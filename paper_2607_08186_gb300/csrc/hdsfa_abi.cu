@@ -76,6 +76,36 @@ hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t m
     g->rs = 1;
     g->window = mode == SFA_LOCAL ? window : 0;
   }
+  // queries are the key rows themselves
+  g->Lq = g->Lv;
+  g->qstep = 1;
+  g->qoff = 0;
+  g->q_nL = g->nL;
+  g->q_ns = g->ns;
+  g->q_rs = g->rs;
+  g->kv_s0 = 0;
+  return HD_OK;
+}
+
+// A final-stream problem: the L final-stream queries (positions t*n + n-1, the rows
+// the loss reads, Eq. 2) in dense [B][L] tensors against the keys of the layer's mask.
+hd_status_t make_final_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, int window,
+                            SfaGeom* g) {
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, g);
+  if (st != HD_OK) return st;
+  g->Lq = L;
+  g->q_nL = L;
+  g->q_ns = 1;
+  g->q_rs = 1;
+  if (mode == SFA_WITHIN) {  // the problem of stream n-1: query row t is its key row t
+    g->qstep = 1;
+    g->qoff = 0;
+    g->kv_s0 = n - 1;
+  } else {  // query row t at position t*n + n-1 of the nL key rows
+    g->qstep = n;
+    g->qoff = n - 1;
+    g->kv_s0 = 0;
+  }
   return HD_OK;
 }
 
@@ -102,15 +132,18 @@ struct BwdWs {
   float* delta;
 };
 
-size_t ws_bytes(const SfaGeom& g, int Dh) {
+// Sizes follow the query side (query_geom): the accumulator and row terms are per query row.
+size_t ws_bytes(const SfaGeom& gk, int Dh) {
+  const SfaGeom g = query_geom(gk);
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
   const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)row_terms_pitch(g.Lv);
   return align256(rows * Dh * sizeof(float)) + 2 * align256(trows * sizeof(float));
 }
 
-hd_status_t split_ws(const SfaGeom& g, int Dh, void* ws, size_t bytes, BwdWs* out) {
-  if (ws == nullptr || bytes < ws_bytes(g, Dh) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+hd_status_t split_ws(const SfaGeom& gk, int Dh, void* ws, size_t bytes, BwdWs* out) {
+  if (ws == nullptr || bytes < ws_bytes(gk, Dh) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
     return HD_ERR_WORKSPACE;
+  const SfaGeom g = query_geom(gk);
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
   const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)row_terms_pitch(g.Lv);
   char* p = static_cast<char*>(ws);
@@ -219,7 +252,7 @@ hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int 
   if (st != HD_OK) return st;
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
-  return cuda_status(hdsfa::launch_sfa_bwd_prep(o, dout, lse, ws.lse2, ws.delta, ws.dq, g, Dh, stream));
+  return cuda_status(hdsfa::launch_sfa_bwd_prep(o, dout, lse, ws.lse2, ws.delta, ws.dq, query_geom(g), Dh, stream));
 }
 
 hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void* dout, void* dk, void* dv,
@@ -252,7 +285,7 @@ hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int
   if (st != HD_OK) return st;
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
-  return cuda_status(hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, g, Dh,
+  return cuda_status(hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, query_geom(g), Dh,
                                                     resolve_scale(softmax_scale, Dh), stream));
 }
 
@@ -322,6 +355,54 @@ hd_status_t sfa_kv_append(const void* k_new, const void* v_new, void* k_cache, v
   if ((long long)Lcap * n > (1LL << 30)) return HD_ERR_UNSUPPORTED;
   return cuda_status(hdsfa::launch_kv_append(k_new, v_new, k_cache, v_cache, lens, B, Lcap, n, Hkv, Dh,
                                              dev_status, stream));
+}
+
+// ---- final-stream problems (Eq. 2 rows; Sec. 3.1 final-stream-only layers) ----
+hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L, int n,
+                          int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
+                          int32_t* dev_status, cudaStream_t stream) {
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
+    return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
+  if (st != HD_OK) return st;
+  if (use_mma_kernels()) return HD_ERR_UNSUPPORTED;  // the mma.sync kernels have no final-stream geometry
+  return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, resolve_scale(softmax_scale, Dh), dev_status,
+                                              stream));
+}
+
+size_t sfa_bwd_final_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode) {
+  SfaGeom g;
+  if (Dh != 128 || make_final_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g) != HD_OK) return 0;
+  return ws_bytes(g, Dh);
+}
+
+hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                          const void* dout, void* dq, void* dk, void* dv, int B, int L, int n, int Hq, int Hkv,
+                          int Dh, float softmax_scale, sfa_mode_t mode, int window, void* workspace,
+                          size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream) {
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
+      !aligned16(dout) || !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+    return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
+  if (st != HD_OK) return st;
+  if (Dh != 128 || use_mma_kernels()) return HD_ERR_UNSUPPORTED;  // the tcgen05 backward is head dim 128
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  const float scale = resolve_scale(softmax_scale, Dh);
+  const SfaGeom gq = query_geom(g);
+  cudaError_t e = hdsfa::launch_sfa_bwd_prep(o, dout, lse, ws.lse2, ws.delta, ws.dq, gq, Dh, stream);
+  if (e == cudaSuccess && mode == SFA_WITHIN) {
+    // only stream n-1's keys are seen by the final-stream queries: the other rows are zero
+    const size_t bytes = (size_t)B * n * L * Hkv * Dh * 2;
+    e = cudaMemsetAsync(dk, 0, bytes, stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dv, 0, bytes, stream);
+  }
+  if (e == cudaSuccess)
+    e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status, stream);
+  if (e == cudaSuccess) e = hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, gq, Dh, scale, stream);
+  return cuda_status(e);
 }
 
 const char* hd_status_string(hd_status_t s) {

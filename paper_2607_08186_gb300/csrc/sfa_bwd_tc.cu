@@ -4,7 +4,8 @@
 // One CTA owns a 128-row key tile j of one virtual causal problem (SfaGeom) and
 // one K/V head; it loops over the group's query heads and over the 128-row query
 // tiles that can see tile j (causal: query tiles at or after the key tile; LOCAL:
-// also within the window).  Every GEMM is a 128 x 128 x 16k tcgen05 MMA (N = 128
+// also within the window; a final-stream problem maps query row r to key row
+// r*qstep + qoff).  Every GEMM is a 128 x 128 x 16k tcgen05 MMA (N = 128
 // runs at full tensor rate; N = 64 does not):
 //   S'^T = K Q^T - lse2/c2 (-inf on masked pairs),  dP'^T = V dO^T - delta
 //                                       SS: A = K / V (K-major), B = Q / dO (K-major),
@@ -91,9 +92,6 @@ struct Params {
   int32_t* status;
 };
 
-HD_DEVINLINE bool visible(int r, int c, int Lv, int window) {
-  return c <= r && r < Lv && c < Lv && (window <= 0 || r - c < window);
-}
 
 __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant__ Params P) {
   extern __shared__ uint8_t smem_raw[];
@@ -111,18 +109,31 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // linear grid, key tile slowest: every CTA of key tile 0 (the most query tiles to
   // visit) launches before any of tile 1, and so on, over all heads, streams and batches
-  const int per_tile = G.Hkv * G.ns * G.B;
+  const int per_tile = G.Hkv * G.q_ns * G.B;
   const int j = (int)blockIdx.x / per_tile;
   const int hsb = (int)blockIdx.x % per_tile;
   const int n0 = j * BK;
-  const int b = hsb / (G.Hkv * G.ns), kvh = (hsb / G.ns) % G.Hkv, s = hsb % G.ns;
+  const int b = hsb / (G.Hkv * G.q_ns), kvh = (hsb / G.q_ns) % G.Hkv, s = hsb % G.q_ns;
+  const int sk = s + G.kv_s0;  // stream of the key problem
   const int grp = G.Hq / G.Hkv;
-  const int i_lo = n0 / BQ;
-  int i_hi = (G.Lv - 1) / BQ;
-  if (G.window > 0) i_hi = min(i_hi, (n0 + BK - 1 + G.window - 1) / BQ);
+  // query rows that can see a key of the tile: key row r*qstep + qoff >= n0, and under
+  // a window r*qstep + qoff < n0 + BK - 1 + window
+  const int i_lo = (n0 <= G.qoff ? 0 : (n0 - G.qoff + G.qstep - 1) / G.qstep) / BQ;
+  int i_hi = (G.Lq - 1) / BQ;
+  if (G.window > 0) i_hi = min(i_hi, ((n0 + BK - 2 + G.window - G.qoff) / G.qstep) / BQ);
   const int nq = i_hi - i_lo + 1;
   const int T = grp * nq;
-  const int Lvp = row_terms_pitch(G.Lv);
+  const int Lqp = row_terms_pitch(G.Lq);
+  if (nq <= 0) {  // no query sees this key tile: its dK and dV rows are zero
+    for (int i = threadIdx.x; i < BK * (DH / 8); i += NTHREADS) {
+      const int kr = n0 + i / (DH / 8), c = i % (DH / 8);
+      if (kr >= G.Lv) continue;
+      const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + sk) * G.Hkv + kvh) * DH + c * 8;
+      *reinterpret_cast<uint4*>(P.dk + orow) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(P.dv + orow) = make_uint4(0, 0, 0, 0);
+    }
+    return;
+  }
 
   if (threadIdx.x == 0) {
     mbar_init(&sm.kv_full, 1);
@@ -167,8 +178,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       tma_prefetch(&P.tm_v);
       mbar_arrive_expect_tx(&sm.kv_full, 2 * BK * DH * 2);
       for (int c = 0; c < DH / 64; ++c) {
-        tma_load_5d(sm.k + c * BK * 64, &P.tm_k, &sm.kv_full, c * 64, kvh, s, n0, b);
-        tma_load_5d(sm.v + c * BK * 64, &P.tm_v, &sm.kv_full, c * 64, kvh, s, n0, b);
+        tma_load_5d(sm.k + c * BK * 64, &P.tm_k, &sm.kv_full, c * 64, kvh, sk, n0, b);
+        tma_load_5d(sm.v + c * BK * 64, &P.tm_v, &sm.kv_full, c * 64, kvh, sk, n0, b);
       }
       int nq_issued = 0, ndo_issued = 0;
       // query tiles (with their row terms) run up to two ahead (double buffer); dO one ahead
@@ -179,7 +190,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         mbar_arrive_expect_tx(&sm.q_full[qb], BQ * DH * 2 + 2 * BQ * 4);
         for (int c = 0; c < DH / 64; ++c)
           tma_load_5d(sm.q[qb] + c * BQ * 64, &P.tm_q, &sm.q_full[qb], c * 64, h, s, q0, b);
-        const long long off = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + q0;
+        const long long off = (((long long)b * G.Hq + h) * G.q_ns + s) * Lqp + q0;
         bulk_load(sm.nlse2[qb], P.lse2 + off, BQ * 4, &sm.q_full[qb]);
         bulk_load(sm.ndelta[qb], P.delta + off, BQ * 4, &sm.q_full[qb]);
         ++nq_issued;
@@ -403,7 +414,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     // epilogue: this key row of dV, then of dK (scaled)
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
       tc_fence_after();
-      const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + s) * G.Hkv + kvh) * DH;
+      const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + sk) * G.Hkv + kvh) * DH;
 #pragma unroll 1
       for (int c = 0; c < 2 * DH / 32; ++c) {
         const int which = c >= DH / 32;
@@ -455,15 +466,21 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         w[4 * i + 2] = __float_as_uint(x.z * inv_c2);
         w[4 * i + 3] = __float_as_uint(x.w * inv_c2);
       }
-      if ((qm < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (qm + BQ > G.Lv)) {
-        // key row kr sees the queries q in [kr, vis_hi): causal, inside the sequence,
-        // and for LOCAL inside the window (an empty range when kr itself is past Lv)
-        const long long lim = G.window > 0 ? min((long long)G.Lv, (long long)kr + G.window) : (long long)G.Lv;
-        const int vis_hi = kr < G.Lv ? (int)lim : kr;
+      if ((qm * G.qstep + G.qoff < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (qm + BQ > G.Lq)) {
+        // key row kr sees the queries q in [vis_lo, vis_hi): q*qstep + qoff >= kr
+        // (causal), q < Lq, and for LOCAL q*qstep + qoff < kr + window (an empty range
+        // when kr itself is past Lv)
+        const int vis_lo = kr <= G.qoff ? 0 : (kr - G.qoff + G.qstep - 1) / G.qstep;
+        int vis_hi = G.Lq;
+        if (G.window > 0) {
+          const int e = kr + G.window - G.qoff;  // q*qstep < e
+          vis_hi = min(vis_hi, e <= 0 ? 0 : (e + G.qstep - 1) / G.qstep);
+        }
+        if (kr >= G.Lv) vis_hi = 0;
         const int qb = qm + 64 * dhalf;
 #pragma unroll
         for (int i = 0; i < 64; ++i)
-          if (qb + i < kr || qb + i >= vis_hi) w[i] = __float_as_uint(-INFINITY);
+          if (qb + i < vis_lo || qb + i >= vis_hi) w[i] = __float_as_uint(-INFINITY);
       }
     };
     auto d_values = [&](uint32_t* w, const float* src) {  // dP'^T: -delta
@@ -581,9 +598,10 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
                                    const SfaGeom& g, float scale, int32_t* status, cudaStream_t st) {
   using namespace tcbwd;
   Params p;
-  if (!make_rows_tmap(&p.tm_q, q, g, g.Hq, DH, BQ) || !make_rows_tmap(&p.tm_do, dout, g, g.Hq, DH, BQ) ||
+  const SfaGeom gq = query_geom(g);
+  if (!make_rows_tmap(&p.tm_q, q, gq, g.Hq, DH, BQ) || !make_rows_tmap(&p.tm_do, dout, gq, g.Hq, DH, BQ) ||
       !make_rows_tmap(&p.tm_k, k, g, g.Hkv, DH, BK) || !make_rows_tmap(&p.tm_v, v, g, g.Hkv, DH, BK) ||
-      !make_rows_tmap(&p.tm_dq, dq_ws, g, g.Hq, DH, 32, 4, 32, true))
+      !make_rows_tmap(&p.tm_dq, dq_ws, gq, g.Hq, DH, 32, 4, 32, true))
     return cudaErrorInvalidValue;
   p.lse2 = lse2_ws;
   p.delta = delta_ws;
@@ -596,7 +614,7 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   const int smem = kSmemBytes;
   cudaError_t e = cudaFuncSetAttribute(bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.ns * g.B);
+  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.q_ns * g.B);
   bwd_kernel<<<grid, NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }

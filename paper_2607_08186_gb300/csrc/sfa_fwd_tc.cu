@@ -5,7 +5,9 @@
 // visits only that stream's key tiles; CROSS is causal over all nL positions
 // (Fig. 2a); LOCAL adds the window (Fig. 2b).  Key tiles past the diagonal (or
 // before the window) are skipped; tiles straddling a mask edge are masked in
-// registers.
+// registers.  A final-stream problem has only the L final-stream queries (dense
+// [B][L] tensors) against the same keys: query row r stands at key row
+// r*qstep + qoff, which sets its tile range and mask.
 //
 // Roles (192 threads):
 //   warp 0      TMA producer: Q once, then K/V tiles into a 2-stage ring; owns TMEM.
@@ -47,19 +49,21 @@ struct Params {
   int32_t* status;
 };
 
-HD_DEVINLINE bool visible(int r, int c, int Lv, int window) {
-  return c <= r && c < Lv && (window <= 0 || r - c < window);
+// Key row c visible from the query at key row rq (= r*qstep + qoff).
+HD_DEVINLINE bool visible(int rq, int c, int Lv, int window) {
+  return c <= rq && c < Lv && (window <= 0 || rq - c < window);
 }
 
 // Key-tile range [lo, hi] of the query tile starting at row m0 (hi < lo: no rows).
 HD_DEVINLINE void tile_range(const SfaGeom& G, int m0, int& lo, int& hi) {
-  if (m0 >= G.Lv) {
+  if (m0 >= G.Lq) {
     lo = 0;
     hi = -1;
     return;
   }
-  lo = G.window > 0 ? max(0, m0 - G.window + 1) / BN : 0;
-  hi = min(m0 / BN, (G.Lv - 1) / BN);
+  const int rq_first = m0 * G.qstep + G.qoff, rq_last = (min(m0 + BM, G.Lq) - 1) * G.qstep + G.qoff;
+  lo = G.window > 0 ? max(0, rq_first - G.window + 1) / BN : 0;
+  hi = min(rq_last / BN, (G.Lv - 1) / BN);
 }
 
 // TMEM columns: S_g at g*128 (P_g packed bf16 over its first 64 columns), O_g at 256 + g*DH.
@@ -69,14 +73,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
   Smem<DH>& sm = *reinterpret_cast<Smem<DH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ncta = (G.Lv + NG * BM - 1) / (NG * BM);
+  const int ncta = (G.Lq + NG * BM - 1) / (NG * BM);
   // linear grid, query-tile rank slowest: the last query tiles (the most key tiles to
   // visit) of every head, stream and batch launch first
-  const int per_rank = G.Hq * G.ns * G.B;
+  const int per_rank = G.Hq * G.q_ns * G.B;
   const int mt = ncta - 1 - (int)blockIdx.x / per_rank;
   const int hsb = (int)blockIdx.x % per_rank;
   const int m0 = mt * NG * BM;
-  const int b = hsb / (G.Hq * G.ns), h = (hsb / G.ns) % G.Hq, s = hsb % G.ns;
+  const int b = hsb / (G.Hq * G.q_ns), h = (hsb / G.q_ns) % G.Hq, s = hsb % G.q_ns;
+  const int sk = s + G.kv_s0;  // stream of the key problem
   const int kvh = h / (G.Hq / G.Hkv);
   int lo[NG], hi[NG];
 #pragma unroll
@@ -127,8 +132,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
         if (it >= NST && !mbar_wait(&sm.kv_empty[st], ((it / NST) - 1) & 1, abort, P.status)) break;
         mbar_arrive_expect_tx(&sm.kv_full[st], 2 * BN * DH * 2);
         for (int c = 0; c < DH / 64; ++c) {
-          tma_load_5d(sm.k[st] + c * BN * 64, &P.tm_k, &sm.kv_full[st], c * 64, kvh, s, j * BN, b);
-          tma_load_5d(sm.v[st] + c * BN * 64, &P.tm_v, &sm.kv_full[st], c * 64, kvh, s, j * BN, b);
+          tma_load_5d(sm.k[st] + c * BN * 64, &P.tm_k, &sm.kv_full[st], c * 64, kvh, sk, j * BN, b);
+          tma_load_5d(sm.v[st] + c * BN * 64, &P.tm_v, &sm.kv_full[st], c * 64, kvh, sk, j * BN, b);
         }
       }
       // every copy this thread started lands before the CTA may exit
@@ -207,6 +212,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
     const int r = m0 + g * BM + row;
+    const int rq = r * G.qstep + G.qoff;                      // its key row
+    const int rq0 = (m0 + g * BM) * G.qstep + G.qoff;         // key row of the tile's first query
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     const uint32_t tS = tl + g * 128, tO = tl + 256 + g * DH;
     const float c2 = P.scale_log2;
@@ -224,11 +231,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
       for (int c = 0; c < BN / 32; ++c) tmem_ld32(tS + c * 32, reinterpret_cast<uint32_t*>(x) + c * 32);
       tmem_ld_wait();
-      const bool need_mask = (j == hi[g] && (j + 1) * BN > m0 + g * BM) || G.window > 0 || (j + 1) * BN > G.Lv;
+      // tiles holding a key past the first query's key row (the diagonal band), any tile
+      // under a window, and the ragged last tile
+      const bool need_mask = (j + 1) * BN - 1 > rq0 || G.window > 0 || (j + 1) * BN > G.Lv;
       if (need_mask) {
 #pragma unroll
         for (int e = 0; e < BN; ++e)
-          if (!visible(r, j * BN + e, G.Lv, G.window)) x[e] = -INFINITY;
+          if (!visible(rq, j * BN + e, G.Lv, G.window)) x[e] = -INFINITY;
       }
       float mx[8];
 #pragma unroll
@@ -285,13 +294,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     if (ok && hi[g] >= lo[g] && __all_sync(0xffffffffu, mbar_wait(&sm.o_done[g], 0, abort, P.status))) {
       tc_fence_after();
       const float inv = 1.f / l_run;
-      bf16* orow = P.o + (((long long)b * G.nL + (long long)r * G.rs + s) * G.Hq + h) * DH;
+      bf16* orow = P.o + (((long long)b * G.q_nL + (long long)r * G.q_rs + s) * G.Hq + h) * DH;
 #pragma unroll
       for (int c = 0; c < DH / 32; ++c) {
         uint32_t o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_ld_wait();
-        if (r < G.Lv) {
+        if (r < G.Lq) {
 #pragma unroll
           for (int e = 0; e < 32; e += 8) {
             uint4 w;
@@ -303,8 +312,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
           }
         }
       }
-      if (r < G.Lv)
-        P.lse[((long long)b * G.Hq + h) * G.nL + (long long)r * G.rs + s] = (m_run * c2 + log2f(l_run)) * kLn2;
+      if (r < G.Lq)
+        P.lse[((long long)b * G.Hq + h) * G.q_nL + (long long)r * G.q_rs + s] = (m_run * c2 + log2f(l_run)) * kLn2;
     }
   }
 
@@ -324,8 +333,8 @@ static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   const int smem = (int)sizeof(tcfwd::Smem<DH>) + 1024;
   cudaError_t e = cudaFuncSetAttribute(tcfwd::fwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const unsigned grid = (unsigned)((p.g.Lv + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM)) *
-                        (unsigned)(p.g.Hq * p.g.ns * p.g.B);
+  const unsigned grid = (unsigned)((p.g.Lq + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM)) *
+                        (unsigned)(p.g.Hq * p.g.q_ns * p.g.B);
   tcfwd::fwd_kernel<DH><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }
@@ -333,7 +342,8 @@ static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
                               const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st) {
   tcfwd::Params p;
-  if (!make_rows_tmap(&p.tm_q, q, g, g.Hq, Dh, tcfwd::BM) || !make_rows_tmap(&p.tm_k, k, g, g.Hkv, Dh, tcfwd::BN) ||
+  if (!make_rows_tmap(&p.tm_q, q, query_geom(g), g.Hq, Dh, tcfwd::BM) ||
+      !make_rows_tmap(&p.tm_k, k, g, g.Hkv, Dh, tcfwd::BN) ||
       !make_rows_tmap(&p.tm_v, v, g, g.Hkv, Dh, tcfwd::BN))
     return cudaErrorInvalidValue;
   p.o = (bf16*)o;
