@@ -13,8 +13,9 @@ The same JSON line also carries: the dominant kernel's roofline, the end-to-end
 number through the C ABI with host buffers, the CPU oracle baseline, and under
 "extras" the CROSS (full cross-stream) layer of the same shape, the expansion-factor
 sweep, the LOCAL (sliding-window) layer at windows of 1024 and 4096 positions, the
-HBM bandwidth of the expansion backward and the final-stream selection, and of the
-decoding step over the expanded KV cache.
+HBM bandwidth of the expansion backward and the final-stream selection and of the
+decoding step over the expanded KV cache, and the final-stream-only layer (the L
+final-stream queries against all nL keys).
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the paper publishes no implementation to run).
@@ -369,6 +370,49 @@ def measure_expansion_backward(dev, hbm_peak: float, V: int = GATHER_V):
     return out
 
 
+def final_pairs(L: int, n: int, mode: int, window: int = 0) -> int:
+    """Visible pairs per (batch, head) of the final-stream problem: query t at position
+    t*n + n-1 sees (t+1)*n keys (CROSS), t+1 (WITHIN: stream n-1 only), or
+    min((t+1)*n, w) (LOCAL)."""
+    if mode == WITHIN:
+        return L * (L + 1) // 2
+    if mode == CROSS:
+        return n * L * (L + 1) // 2
+    return sum(min((t + 1) * n, window) for t in range(L))
+
+
+def measure_final_layer(dev, bf16_peak: float, iters: int = 5):
+    """Final-stream-only layer (Sec. 3.1 KV-mirror layers: the L final-stream queries against
+    all nL keys), Qwen3-8B-class heads, L=4096, n=4: fwd and bwd TFLOP/s over visible pairs."""
+    from paper_2607_08186_gb300 import binding
+    B, L, n, Hq, Hkv, Dh = 1, 4096, 4, 32, 8, 128
+    g = torch.Generator(device=dev)
+    g.manual_seed(51)
+
+    def rnd(*shape):
+        return torch.randn(*shape, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    q, do = rnd(B, L, Hq, Dh), rnd(B, L, Hq, Dh)
+    k, v = rnd(B, n * L, Hkv, Dh), rnd(B, n * L, Hkv, Dh)
+    o, lse = torch.empty_like(q), torch.empty(B, Hq, L, dtype=torch.float32, device=dev)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    out = {"workload": f"final-stream layer B={B} L={L} n={n} ({n * L} key positions) Hq={Hq} Hkv={Hkv} Dh={Dh}"}
+    for mode in (WITHIN, CROSS):
+        ws = torch.empty(binding.sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
+                         device=dev)
+        tf = time_op(lambda k_: binding.sfa_fwd_final(q, k, v, o, lse, mode), 1, iters=iters)
+        tb = time_op(lambda k_: binding.sfa_bwd_final(q, k, v, o, lse, do, dq, dk, dv, mode, ws), 1, iters=iters)
+        pairs = final_pairs(L, n, mode) * Hq * B
+        out[MODE_NAME[mode]] = {"fwd_ms": tf * 1e3, "bwd_ms": tb * 1e3,
+                                "fwd_tflops": FWD_FLOP * Dh * pairs / tf / 1e12,
+                                "bwd_tflops": BWD_FLOP * Dh * pairs / tb / 1e12,
+                                "fwd_frac": FWD_FLOP * Dh * pairs / tf / 1e12 / bf16_peak,
+                                "bwd_frac": BWD_FLOP * Dh * pairs / tb / 1e12 / bf16_peak}
+    del q, do, k, v, o, lse, dq, dk, dv
+    torch.cuda.empty_cache()
+    return out
+
+
 def measure_decode(dev, hbm_peak: float, quick: bool = False):
     """Decoding step (Sec. 3.2) with Qwen3-8B-class heads (Hq=32, Hkv=8, Dh=128), n=4:
     the new token's 4 positions against a context of T tokens (4T cached positions) for
@@ -516,6 +560,8 @@ def main():
     ap.add_argument("--no-extras", action="store_true", help="skip the extras (CROSS / LOCAL layers, n sweep, expansion backward) and the CPU baseline")
     ap.add_argument("--expand-bwd-only", action="store_true",
                     help="time only the expansion backward and final-stream selection (JSON line)")
+    ap.add_argument("--final-only", action="store_true",
+                    help="time only the final-stream-only layer (JSON line)")
     ap.add_argument("--decode-only", action="store_true",
                     help="time only the decoding step over the serving grid (JSON line)")
     ap.add_argument("--vocab", type=int, default=GATHER_V,
@@ -539,6 +585,11 @@ def main():
     barrier(ws)
     s = SHAPES[WORKLOAD]
     pk = peaks()
+    if args.final_only:
+        r = measure_final_layer(dev, pk["bf16"], iters=args.steps)
+        if rank == 0:
+            print(json.dumps(r), flush=True)
+        return
     if args.decode_only:
         r = measure_decode(dev, pk["hbm"])
         if rank == 0:
@@ -658,6 +709,7 @@ def main():
         extras["local_layer"] = {"workload": f"{WORKLOAD}_local", "windows": loc}
         extras["expansion_backward"] = measure_expansion_backward(dev, pk["hbm"])
         extras["decode"] = measure_decode(dev, pk["hbm"], quick=True)
+        extras["final_stream_layer"] = measure_final_layer(dev, pk["bf16"])
         out["extras"] = extras
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
