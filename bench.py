@@ -14,8 +14,9 @@ number through the C ABI with host buffers, the CPU oracle baseline, and under
 "extras" the CROSS (full cross-stream) layer of the same shape, the expansion-factor
 sweep, the LOCAL (sliding-window) layer at windows of 1024 and 4096 positions, the
 HBM bandwidth of the expansion backward and the final-stream selection and of the
-decoding step over the expanded KV cache, and the final-stream-only layer (the L
-final-stream queries against all nL keys).
+decoding step over the expanded KV cache, the final-stream-only layer (the L
+final-stream queries against all nL keys), and the large-MoE-class stack (L=8192,
+n=4, Hq=64: 7 WITHIN + 1 CROSS layers, forward + backward).
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the paper publishes no implementation to run).
@@ -370,6 +371,65 @@ def measure_expansion_backward(dev, hbm_peak: float, V: int = GATHER_V):
     return out
 
 
+def measure_moe_stack(dev, pk, steps: int = 3, warmup: int = 1):
+    """Large-MoE-class attention stack: B=1, L=8192 tokens, n=4 (32768 positions), Hq=64,
+    Hkv=8, Dh=128; 7 WITHIN layers then 1 CROSS layer, forward + backward of every layer
+    with its own Q, K, V, dO (device-generated N(0,1)).  TMFLOP/s over visible pairs of the
+    whole stack, per step; each layer's inputs and outputs are > 0.5 GB (beyond L2)."""
+    from paper_2607_08186_gb300 import binding
+    s = AttnShape(1, 8192, 4, 64, 8, 128)
+    modes = [WITHIN] * 7 + [CROSS]
+    g = torch.Generator(device=dev)
+    g.manual_seed(61)
+
+    def rnd(*shape):
+        return torch.randn(*shape, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    layers = []
+    for mode in modes:
+        q, k, v, do = rnd(s.B, s.nL, s.Hq, s.Dh), rnd(s.B, s.nL, s.Hkv, s.Dh), rnd(s.B, s.nL, s.Hkv, s.Dh), \
+            rnd(s.B, s.nL, s.Hq, s.Dh)
+        t = {"mode": mode, "q": q, "k": k, "v": v, "do": do, "o": torch.empty_like(q),
+             "lse": torch.empty(s.B, s.Hq, s.nL, dtype=torch.float32, device=dev),
+             "dq": torch.empty_like(q), "dk": torch.empty_like(k), "dv": torch.empty_like(v),
+             "ws": torch.empty(binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),
+                               dtype=torch.uint8, device=dev)}
+        layers.append(t)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(modes) + 1)] for _ in range(steps)]
+
+    def run(ev=None):
+        for i, t in enumerate(layers):
+            if ev is not None:
+                ev[i].record()
+            binding.sfa_fwd(t["q"], t["k"], t["v"], t["o"], t["lse"], s.n, t["mode"])
+            binding.sfa_bwd(t["q"], t["k"], t["v"], t["o"], t["lse"], t["do"], t["dq"], t["dk"], t["dv"], s.n,
+                            t["mode"], t["ws"])
+        if ev is not None:
+            ev[-1].record()
+
+    for _ in range(warmup):
+        run()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for i in range(steps):
+        run(evs[i])
+    t1.record()
+    torch.cuda.synchronize()
+    sec = t0.elapsed_time(t1) / 1e3 / steps
+    flops = sum(attn_flops(s, m, FWD_FLOP + BWD_FLOP) for m in modes)
+    within_ms = statistics.mean(e[i].elapsed_time(e[i + 1]) for e in evs for i in range(7))
+    cross_ms = statistics.mean(e[7].elapsed_time(e[8]) for e in evs)
+    del layers
+    torch.cuda.empty_cache()
+    return {"workload": "moe_large_n4 stack: B=1 L=8192 n=4 (32768 positions) Hq=64 Hkv=8 Dh=128, "
+                        "7 WITHIN + 1 CROSS layers, fwd+bwd (prep, main, finalize) per layer",
+            "ms_per_stack": sec * 1e3, "flops_per_stack": flops, "tflops": flops / sec / 1e12,
+            "frac": flops / sec / 1e12 / pk["bf16"], "frac_of_sustained": flops / sec / 1e12 / pk["bf16_sustained"],
+            "within_layer_ms": within_ms, "within_layer_tflops": attn_flops(s, WITHIN, 14) / within_ms / 1e9,
+            "cross_layer_ms": cross_ms, "cross_layer_tflops": attn_flops(s, CROSS, 14) / cross_ms / 1e9}
+
+
 def final_pairs(L: int, n: int, mode: int, window: int = 0) -> int:
     """Visible pairs per (batch, head) of the final-stream problem: query t at position
     t*n + n-1 sees (t+1)*n keys (CROSS), t+1 (WITHIN: stream n-1 only), or
@@ -560,6 +620,8 @@ def main():
     ap.add_argument("--no-extras", action="store_true", help="skip the extras (CROSS / LOCAL layers, n sweep, expansion backward) and the CPU baseline")
     ap.add_argument("--expand-bwd-only", action="store_true",
                     help="time only the expansion backward and final-stream selection (JSON line)")
+    ap.add_argument("--moe-only", action="store_true",
+                    help="time only the large-MoE-class 8-layer stack (JSON line)")
     ap.add_argument("--final-only", action="store_true",
                     help="time only the final-stream-only layer (JSON line)")
     ap.add_argument("--decode-only", action="store_true",
@@ -585,6 +647,11 @@ def main():
     barrier(ws)
     s = SHAPES[WORKLOAD]
     pk = peaks()
+    if args.moe_only:
+        r = measure_moe_stack(dev, pk, steps=args.steps if args.steps < 20 else 3)
+        if rank == 0:
+            print(json.dumps(r), flush=True)
+        return
     if args.final_only:
         r = measure_final_layer(dev, pk["bf16"], iters=args.steps)
         if rank == 0:
@@ -710,6 +777,7 @@ def main():
         extras["expansion_backward"] = measure_expansion_backward(dev, pk["hbm"])
         extras["decode"] = measure_decode(dev, pk["hbm"], quick=True)
         extras["final_stream_layer"] = measure_final_layer(dev, pk["bf16"])
+        extras["moe_stack"] = measure_moe_stack(dev, pk)
         out["extras"] = extras
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
