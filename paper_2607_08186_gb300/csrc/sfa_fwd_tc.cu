@@ -142,16 +142,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // The whole warp runs the loop (warp-uniform operands); one elected lane issues.
+    {
       constexpr uint32_t idS = idesc_bf16(BM, BN, 0, 0);  // S[q][kv] = Q K^T (both K-major)
       constexpr uint32_t idO = idesc_bf16(BM, DH, 0, 1);  // O[q][d] += P V   (P in TMEM, V MN-major)
       int ps[NG] = {0, 0};                                  // per-group P phases consumed
-      bool ok = mbar_wait(&sm.q_full, 0, abort, P.status);
+      bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.q_full, 0, abort, P.status));
       int kv_ready = n_lo - 1;                              // highest key tile known loaded
       auto wait_kv = [&](int j) -> bool {
         if (j <= kv_ready) return true;
         const int it = j - n_lo;
-        if (!mbar_wait(&sm.kv_full[it % NST], (it / NST) & 1, abort, P.status)) return false;
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.kv_full[it % NST], (it / NST) & 1, abort, P.status))) return false;
         kv_ready = j;
         tc_fence_after();
         return true;
@@ -169,18 +170,18 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
           const uint64_t off = (uint64_t)((kk >> 2) * (128 * 128 / 16) + (kk & 3) * 2);
-          tc_mma_ss(tmem + g * 128, qd + off, kd + off, idS, kk > 0 ? 1u : 0u);
+          tc_mma_ss_w(tmem + g * 128, qd + off, kd + off, idS, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&sm.s_full[g]);
+        tc_commit_w(&sm.s_full[g]);
       };
       auto issue_pv = [&](int g, int j) -> bool {
-        if (!mbar_wait(&sm.p_full[g], ps[g] & 1, abort, P.status)) return false;
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.p_full[g], ps[g] & 1, abort, P.status))) return false;
         ++ps[g];
         tc_fence_after();
         const uint64_t vd = ((j - n_lo) & 1) ? vM1 : vM0;
 #pragma unroll
         for (int kk = 0; kk < BN / 16; ++kk)
-          tc_mma_ts(tmem + 256 + g * DH, tmem + g * 128 + kk * 8, vd + (uint64_t)(kk * 16 * 128 / 16), idO,
+          tc_mma_ts_w(tmem + 256 + g * DH, tmem + g * 128 + kk * 8, vd + (uint64_t)(kk * 16 * 128 / 16), idO,
                     (j > lo[g] || kk > 0) ? 1u : 0u);
         return true;
       };
@@ -191,7 +192,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
           for (int g = 0; ok && g < NG; ++g) {
             if (lo[g] <= j && j <= hi[g]) {
               if (!issue_pv(g, j)) { ok = false; break; }
-              if (j == hi[g]) tc_commit(&sm.o_done[g]);
+              if (j == hi[g]) tc_commit_w(&sm.o_done[g]);
             }
             // S of the next tile for this group reuses its S/P columns: issued after its PV
             if (j + 1 <= hi[g] && lo[g] <= j + 1) {
@@ -199,11 +200,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
               issue_s(g, j + 1);
             }
           }
-          tc_commit(&sm.kv_empty[(j - n_lo) % NST]);
+          tc_commit_w(&sm.kv_empty[(j - n_lo) % NST]);
         }
       }
       // every MMA issued above completes before TMEM / smem are released
-      tc_commit(&sm.drain);
+      tc_commit_w(&sm.drain);
       mbar_drain(&sm.drain, 0);
     }
   } else {
