@@ -192,7 +192,11 @@ class HotPath:
             self.x = torch.empty(s.B, s.nL, GATHER_D, dtype=torch.bfloat16, device=dev)
         self.host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
                          for t in (self.o, self.lse, self.dq, self.dk, self.dv)]
-        self.launches_per_step = 4 + (1 if with_gather else 0)
+        # the dQ accumulator is cleared on a side stream beside the forward (it needs
+        # nothing from it), after the previous step's finalize has read it
+        self.side = torch.cuda.Stream(device=dev)
+        self.ev_clear, self.ev_fin = torch.cuda.Event(), torch.cuda.Event()
+        self.launches_per_step = 5 + (1 if with_gather else 0)
 
     def _bufs(self):
         return {"q": self.q, "k": self.k, "v": self.v, "do": self.do, "ids": getattr(self, "ids", None),
@@ -201,6 +205,10 @@ class HotPath:
     def step(self, ev=None, bufs=None, stream=None):
         b, s = self.b, self.s
         t = bufs or self._bufs()
+        main = stream if stream is not None else torch.cuda.current_stream()
+        self.side.wait_event(self.ev_fin)  # the previous finalize has read the accumulator
+        b.sfa_bwd_clear(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, self.mode, self.ws, stream=self.side)
+        self.ev_clear.record(self.side)
         if self.with_gather:
             b.hd_expand_embed(self.tables, t["ids"], self.x, stream=stream)
         if ev is not None:
@@ -208,7 +216,8 @@ class HotPath:
         b.sfa_fwd(t["q"], t["k"], t["v"], t["o"], t["lse"], s.n, self.mode, window=self.window, stream=stream)
         if ev is not None:
             ev[1].record()
-        b.sfa_bwd_prep(t["o"], t["do"], t["lse"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
+        b.sfa_bwd_row_terms(t["o"], t["do"], t["lse"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
+        main.wait_event(self.ev_clear)
         if ev is not None:
             ev[2].record()
         b.sfa_bwd_main(t["q"], t["k"], t["v"], t["do"], t["dk"], t["dv"], s.n, self.mode, self.ws,
@@ -216,6 +225,7 @@ class HotPath:
         if ev is not None:
             ev[3].record()
         b.sfa_bwd_finalize(t["dq"], s.n, self.mode, self.ws, s.Hkv, stream=stream)
+        self.ev_fin.record(main)
 
     def e2e(self, steps: int, warmup: int, ws: int) -> float:
         """Seconds per step end to end with host buffers: every step copies its inputs

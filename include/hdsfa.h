@@ -164,10 +164,21 @@ hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, 
  *                      into the accumulator and write dk, dv (overwritten).
  *   sfa_bwd_finalize : dq = bf16(scale * accumulator).
  * A later phase reads what the earlier one left in the workspace.
+ * sfa_bwd_prep is itself the two halves below, for a caller that overlaps them:
+ *   sfa_bwd_row_terms: the delta and lse terms only (needs o, so after sfa_fwd);
+ *   sfa_bwd_clear    : only the zeroing of the dQ accumulator.  It needs nothing from
+ *                      the forward, so it may run on another stream beside sfa_fwd,
+ *                      ordered after the previous sfa_bwd_finalize that read the same
+ *                      workspace and before sfa_bwd_main.
  */
 hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int B, int L, int n, int Hq,
                          int Hkv, int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
                          cudaStream_t stream);
+hd_status_t sfa_bwd_row_terms(const void* o, const void* dout, const float* lse, int B, int L, int n,
+                              int Hq, int Hkv, int Dh, sfa_mode_t mode, void* workspace,
+                              size_t workspace_bytes, cudaStream_t stream);
+hd_status_t sfa_bwd_clear(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, void* workspace,
+                          size_t workspace_bytes, cudaStream_t stream);
 hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void* dout, void* dk, void* dv,
                          int B, int L, int n, int Hq, int Hkv, int Dh, float softmax_scale,
                          sfa_mode_t mode, int window, void* workspace, size_t workspace_bytes,

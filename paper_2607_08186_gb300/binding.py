@@ -75,6 +75,10 @@ def lib():
             L.sfa_bwd.argtypes = [P, P, P, P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
             L.sfa_bwd_prep.restype = I
             L.sfa_bwd_prep.argtypes = [P, P, P, I, I, I, I, I, I, I, P, Z, P]
+            L.sfa_bwd_row_terms.restype = I
+            L.sfa_bwd_row_terms.argtypes = [P, P, P, I, I, I, I, I, I, I, P, Z, P]
+            L.sfa_bwd_clear.restype = I
+            L.sfa_bwd_clear.argtypes = [I, I, I, I, I, I, I, P, Z, P]
             L.sfa_bwd_main.restype = I
             L.sfa_bwd_main.argtypes = [P, P, P, P, P, P, I, I, I, I, I, I, F, I, I, P, Z, P, P]
             L.sfa_bwd_finalize.restype = I
@@ -291,6 +295,19 @@ def sfa_bwd_prep(o, dout, lse, n, mode, workspace, Hkv, stream=None):
     B, nL, Hq, Dh = o.shape
     _check(lib().sfa_bwd_prep(_p(o), _p(dout), _p(lse), B, nL // n, n, Hq, Hkv, Dh, int(mode),
                               _p(workspace), _wsb(workspace), _stream(stream)), "sfa_bwd_prep")
+
+
+def sfa_bwd_row_terms(o, dout, lse, n, mode, workspace, Hkv, stream=None):
+    """The delta / lse half of sfa_bwd_prep (no zeroing of the dQ accumulator)."""
+    B, nL, Hq, Dh = o.shape
+    _check(lib().sfa_bwd_row_terms(_p(o), _p(dout), _p(lse), B, nL // n, n, Hq, Hkv, Dh, int(mode),
+                                   _p(workspace), _wsb(workspace), _stream(stream)), "sfa_bwd_row_terms")
+
+
+def sfa_bwd_clear(B, L, n, Hq, Hkv, Dh, mode, workspace, stream=None):
+    """The other half: zero the workspace's fp32 dQ accumulator (independent of the forward)."""
+    _check(lib().sfa_bwd_clear(B, L, n, Hq, Hkv, Dh, int(mode), _p(workspace), _wsb(workspace),
+                               _stream(stream)), "sfa_bwd_clear")
 
 
 def sfa_bwd_main(q, k, v, dout, dk, dv, n, mode, workspace, softmax_scale=0.0, window=0,

@@ -33,7 +33,8 @@ cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void
                                const SfaGeom& g, int Dh, float scale, cudaStream_t st);
 cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
                                 float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
-                                cudaStream_t st);
+                                cudaStream_t st, bool zero = true);
+cudaError_t launch_sfa_bwd_clear(float* dq_ws, const SfaGeom& g, int Dh, cudaStream_t st);
 cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const void* dout,
                                     void* dk, void* dv, const float* lse2_ws, const float* delta_ws,
                                     float* dq_ws, const SfaGeom& g, int Dh, float scale,
@@ -253,6 +254,29 @@ hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int 
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
   return cuda_status(hdsfa::launch_sfa_bwd_prep(o, dout, lse, ws.lse2, ws.delta, ws.dq, query_geom(g), Dh, stream));
+}
+
+hd_status_t sfa_bwd_row_terms(const void* o, const void* dout, const float* lse, int B, int L, int n, int Hq,
+                              int Hkv, int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
+                              cudaStream_t stream) {
+  if (!aligned16(o) || !aligned16(dout) || !aligned16(lse)) return HD_ERR_INVALID_ARG;
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
+  if (st != HD_OK) return st;
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  return cuda_status(
+      hdsfa::launch_sfa_bwd_prep(o, dout, lse, ws.lse2, ws.delta, ws.dq, query_geom(g), Dh, stream, false));
+}
+
+hd_status_t sfa_bwd_clear(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, void* workspace,
+                          size_t workspace_bytes, cudaStream_t stream) {
+  SfaGeom g;
+  hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
+  if (st != HD_OK) return st;
+  BwdWs ws;
+  if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
+  return cuda_status(hdsfa::launch_sfa_bwd_clear(ws.dq, query_geom(g), Dh, stream));
 }
 
 hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void* dout, void* dk, void* dv,

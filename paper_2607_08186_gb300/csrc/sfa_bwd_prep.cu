@@ -6,7 +6,8 @@
 //           of any stream is contiguous floats (a single bulk copy).  Negated so the
 //           backward folds them in with one add / fused multiply-add.  Rows in
 //           [Lv, Lvp) get -lse2 = -inf and -delta = 0 (their P and dS vanish).
-//           Also zeroes the fp32 dQ accumulator.
+//           Also zeroes the fp32 dQ accumulator (or leaves that to clear, which needs
+//           nothing from the forward and may run beside it on another stream).
 // finalize: dq = bf16(scale * accumulator), round to nearest even.
 #include "common.cuh"
 
@@ -16,9 +17,9 @@ typedef __nv_bfloat16 bf16;
 
 // One warp takes RPW consecutive (b, p, h) rows: DH/8 lanes per row (16 bytes of O and
 // of dO each), 32*8/DH rows side by side, ITER such row groups with every load issued
-// before the first dot product, so each warp keeps several KB in flight.  The warp
-// then zeroes the same rows of the fp32 dQ accumulator (contiguous, 16-byte stores).
-template <int DH>
+// before the first dot product, so each warp keeps several KB in flight.  With ZERO the
+// warp then zeroes the same rows of the fp32 dQ accumulator (contiguous, 16-byte stores).
+template <int DH, bool ZERO>
 __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restrict__ o,
                                                            const bf16* __restrict__ dout,
                                                            const float* __restrict__ lse,
@@ -64,10 +65,17 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
       lse2_t[t] = -lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
     }
   }
-  // zero dQ accumulator rows [row0, row0 + RPW): RPW * DH floats, contiguous
-  const long long nz = (min(nrows, row0 + RPW) - row0) * DH / 4;
-  float4* dz = reinterpret_cast<float4*>(dq_acc + row0 * DH);
-  for (long long c = lane; c < nz; c += 32) dz[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (ZERO) {  // zero dQ accumulator rows [row0, row0 + RPW): RPW * DH floats, contiguous
+    const long long nz = (min(nrows, row0 + RPW) - row0) * DH / 4;
+    float4* dz = reinterpret_cast<float4*>(dq_acc + row0 * DH);
+    for (long long c = lane; c < nz; c += 32) dz[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+
+// The fp32 dQ accumulator alone, zeroed with 16-byte stores (grid-stride).
+__global__ void __launch_bounds__(256) sfa_bwd_clear_kernel(float4* __restrict__ acc, long long n4) {
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (long long)gridDim.x * blockDim.x)
+    acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 __global__ void sfa_bwd_pad_kernel(float* __restrict__ lse2_t, float* __restrict__ delta_t, SfaGeom g) {
@@ -96,17 +104,23 @@ __global__ void __launch_bounds__(256) sfa_bwd_finalize_kernel(const float* __re
 
 cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
                                 float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
-                                cudaStream_t st) {
+                                cudaStream_t st, bool zero) {
   const long long rows = (long long)g.B * g.nL * g.Hq;
   const long long rpw = 4LL * (32 / (Dh / 8));  // rows per warp (ITER * rows per group)
   const long long warps = (rows + rpw - 1) / rpw;
   const unsigned blocks = (unsigned)((warps * 32 + 255) / 256);
-  if (Dh == 64)
-    sfa_bwd_prep_kernel<64><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, lse, lse2_ws,
-                                                   delta_ws, dq_ws, g);
-  else
-    sfa_bwd_prep_kernel<128><<<blocks, 256, 0, st>>>((const bf16*)o, (const bf16*)dout, lse, lse2_ws,
-                                                    delta_ws, dq_ws, g);
+  const bf16 *ob = (const bf16*)o, *db = (const bf16*)dout;
+  if (Dh == 64) {
+    if (zero)
+      sfa_bwd_prep_kernel<64, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+    else
+      sfa_bwd_prep_kernel<64, false><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+  } else {
+    if (zero)
+      sfa_bwd_prep_kernel<128, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+    else
+      sfa_bwd_prep_kernel<128, false><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int pad = row_terms_pitch(g.Lv) - g.Lv;
@@ -116,6 +130,14 @@ cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* ls
     e = cudaGetLastError();
   }
   return e;
+}
+
+cudaError_t launch_sfa_bwd_clear(float* dq_ws, const SfaGeom& g, int Dh, cudaStream_t st) {
+  const long long n4 = (long long)g.B * g.nL * g.Hq * Dh / 4;
+  long long blocks = (n4 + 255) / 256;
+  if (blocks > 152LL * 16) blocks = 152LL * 16;
+  sfa_bwd_clear_kernel<<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<float4*>(dq_ws), n4);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,

@@ -9,15 +9,18 @@
 // [B][L] tensors) against the same keys: query row r stands at key row
 // r*qstep + qoff, which sets its tile range and mask.
 //
-// Roles (192 threads):
-//   warp 0      TMA producer: Q once, then K/V tiles into a 2-stage ring; owns TMEM.
-//   warp 1      MMA issuer (one thread): S = Q K^T into one of two TMEM S buffers,
-//               O += P V into the TMEM O accumulator.
-//   warps 2..5  softmax: one thread per query row (its TMEM lane); online softmax
-//               in fp32 with exp2, P (bf16) to shared memory, O rescaled in TMEM
-//               only when the running max grows by more than 2^8, epilogue.
-// Shared-memory tiles use the 128-byte swizzle written by TMA; P is written by
-// the softmax threads in the same layout.  Every mbarrier wait is bounded.
+// Roles (320 threads; a CTA owns two 128-row query tiles, groups g = 0, 1):
+//   warp 0      TMA producer: both Q tiles once, then K/V tiles into a 2-stage ring;
+//               owns TMEM.
+//   warp 1      MMA issuer: the whole warp runs the issue loop, one elected lane
+//               issues.  Per key tile and group: S_g = Q_g K^T (SS) into the group's
+//               128 TMEM columns, O_g += P_g V (TS: P_g read from TMEM) into its O
+//               columns; the next S_g is issued after the PV that reads P_g.
+//   warps 2..5, 6..9  softmax of group 0 / 1: one thread per query row (its TMEM
+//               lane); online softmax in fp32 with exp2 (packed f32x2 arithmetic),
+//               P packed to bf16 over the first 64 columns of S_g, O_g rescaled in
+//               TMEM only when the running max grows by more than 2^8, epilogue.
+// K/V tiles use the 128-byte swizzle written by TMA.  Every mbarrier wait is bounded.
 #include "tc_common.cuh"
 
 namespace hdsfa {

@@ -85,6 +85,40 @@ def test_deterministic_forward():
     assert torch.equal(a[3], b[3]) and torch.equal(a[4], b[4])
 
 
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_prep_halves_with_the_clear_on_a_side_stream(mode):
+    # sfa_bwd_row_terms on the main stream, sfa_bwd_clear on another (workspace filled
+    # with NaN bytes first), then main + finalize: the oracle's gradients, and dK / dV
+    # bit-identical to the one-call sfa_bwd
+    s = AttnShape(1, 300, 4, 8, 2, 128)
+    q, k, v, do = inputs.attn_inputs(s, seed=14)
+    qd, kd, vd, dod = q.cuda(), k.cuda(), v.cuda(), do.cuda()
+    o = torch.empty_like(qd)
+    lse = torch.empty(s.B, s.Hq, s.nL, dtype=torch.float32, device="cuda")
+    binding.sfa_fwd(qd, kd, vd, o, lse, s.n, mode)
+    ws = torch.full((binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),), 255,
+                    dtype=torch.uint8, device="cuda")
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        binding.sfa_bwd_clear(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode, ws, stream=side)
+        cleared = torch.cuda.Event()
+        cleared.record(side)
+    binding.sfa_bwd_row_terms(o, dod, lse, s.n, mode, ws, s.Hkv)
+    torch.cuda.current_stream().wait_event(cleared)
+    dq, dk, dv = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
+    binding.sfa_bwd_main(qd, kd, vd, dod, dk, dv, s.n, mode, ws)
+    binding.sfa_bwd_finalize(dq, s.n, mode, ws, s.Hkv)
+    dq1, dk1, dv1 = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
+    ws1 = torch.empty_like(ws)
+    binding.sfa_bwd(qd, kd, vd, o, lse, dod, dq1, dk1, dv1, s.n, mode, ws1)
+    torch.cuda.synchronize()
+    dq_r, dk_r, dv_r = oracle.sfa_bwd(q, k, v, do, s.n, mode)
+    assert_grads_close([("dq", dq.cpu(), dq_r), ("dk", dk.cpu(), dk_r), ("dv", dv.cpu(), dv_r)])
+    assert torch.equal(dk.view(torch.int16), dk1.view(torch.int16))
+    assert torch.equal(dv.view(torch.int16), dv1.view(torch.int16))
+
+
 # ------------------------------------------------------------ full-size layers
 def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
     q, k, v, do = inputs.attn_inputs(s, seed=seed)
