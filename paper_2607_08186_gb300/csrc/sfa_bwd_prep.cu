@@ -31,6 +31,8 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
   constexpr int ITER = 4;            // row groups per warp
   constexpr int RPW = RPG * ITER;    // rows per warp
   const int lane = threadIdx.x & 31, sub = lane / LPR, l = lane % LPR;
+  // row indices fit 32 bits (the host caps B*nL*Hq below 2^30): 32-bit index math, whose
+  // divisions cost a fraction of 64-bit ones
   const long long nrows = (long long)g.B * g.nL * g.Hq;
   const long long row0 = (((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * RPW;
   if (row0 >= nrows) return;
@@ -58,11 +60,12 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
     for (int off = LPR / 2; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
     const long long row = row0 + i * RPG + sub;
     if (l == 0 && row < nrows) {
-      const long long h = row % g.Hq, bp = row / g.Hq, p = bp % g.nL, b = bp / g.nL;
-      const long long s = p % g.ns, r = p / g.ns;
-      const long long t = ((b * g.Hq + h) * g.ns + s) * Lvp + r;
+      const unsigned ur = (unsigned)row, Hq = (unsigned)g.Hq, nL = (unsigned)g.nL, ns = (unsigned)g.ns;
+      const unsigned bp = ur / Hq, h = ur - bp * Hq, b = bp / nL, p = bp - b * nL;
+      const unsigned r = p / ns, s = p - r * ns;
+      const long long t = (((long long)b * Hq + h) * ns + s) * Lvp + r;
       delta_t[t] = -acc;
-      lse2_t[t] = -lse[(b * g.Hq + h) * g.nL + p] * 1.4426950408889634f;
+      lse2_t[t] = -lse[((long long)b * Hq + h) * nL + p] * 1.4426950408889634f;
     }
   }
   if (ZERO) {  // zero dQ accumulator rows [row0, row0 + RPW): RPW * DH floats, contiguous
