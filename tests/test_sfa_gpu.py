@@ -56,6 +56,14 @@ def test_sweep(shape, mode):
     _full_case(AttnShape(*shape), mode, seed=11 + sum(shape))
 
 
+@pytest.mark.parametrize("mode,window", [(WITHIN, 0), (CROSS, 0), (LOCAL, 77)])
+def test_wide_gqa_groups(mode, window):
+    # the paper's 617B head layout (96 query heads over 8 K/V heads: 12 per group) and
+    # a 3-head group (Hq=6, Hkv=2), B=2, ragged nL = 4 * 150 = 600
+    _full_case(AttnShape(1, 150, 4, 96, 8, 128), mode, seed=21, window=window)
+    _full_case(AttnShape(2, 150, 4, 6, 2, 128), mode, seed=22, window=window)
+
+
 @pytest.mark.parametrize("window", [1, 50, 200])
 def test_local_window(window):
     _full_case(AttnShape(1, 96, 4, 4, 2, 128), LOCAL, seed=5, window=window)
