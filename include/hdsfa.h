@@ -36,7 +36,7 @@ extern "C" {
 typedef enum {
   HD_OK = 0,
   HD_ERR_INVALID_ARG = 1, /* null / misaligned pointer, non-positive size, Hq % Hkv != 0 */
-  HD_ERR_UNSUPPORTED = 2, /* valid but not implemented (e.g. Dh not in {64, 128}) */
+  HD_ERR_UNSUPPORTED = 2, /* valid but not implemented (e.g. Dh not in {64, 128, 256}) */
   HD_ERR_CUDA = 3,        /* a CUDA runtime/driver call or kernel launch failed */
   HD_ERR_WORKSPACE = 4,   /* workspace null or smaller than sfa_bwd_workspace_bytes() */
   HD_ERR_TIMEOUT = 5,     /* reserved: a bounded device wait expired (see HD_DEVBIT_TIMEOUT) */
@@ -126,7 +126,9 @@ hd_status_t hd_select_final_stream_bwd(const void* dy, void* dx, int B, int L, i
  *   lse[b][h][p] = log sum_{p' visible} exp(scale * q_p . k_p').
  * q: bf16 [B][nL][Hq][Dh]; k, v: bf16 [B][nL][Hkv][Dh]; o: bf16 like q (written);
  * lse: float32 [B][Hq][nL] (written).  softmax_scale <= 0 selects 1/sqrt(Dh).
- * window is used only by SFA_LOCAL (must be >= 1 there).  Dh in {64, 128}.
+ * window is used only by SFA_LOCAL (must be >= 1 there).  Dh in {64, 128, 256}: 128 runs
+ * on the tcgen05 kernels, 64 (backward) and 256 (the paper's 80B configuration, Table 6)
+ * on warp-level mma.sync kernels.
  * Every position sees itself, so no softmax row is empty.
  */
 hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,

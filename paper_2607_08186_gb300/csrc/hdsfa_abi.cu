@@ -57,7 +57,7 @@ hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t m
   if (Hq % Hkv != 0) return HD_ERR_INVALID_ARG;
   if (mode != SFA_WITHIN && mode != SFA_CROSS && mode != SFA_LOCAL) return HD_ERR_INVALID_ARG;
   if (mode == SFA_LOCAL && window <= 0) return HD_ERR_INVALID_ARG;
-  if (Dh != 64 && Dh != 128) return HD_ERR_UNSUPPORTED;
+  if (Dh != 64 && Dh != 128 && Dh != 256) return HD_ERR_UNSUPPORTED;
   const long long nL = (long long)n * L;
   // Every row index, head product and tile count must fit the kernels' int math.
   if (nL > (1LL << 30) || (long long)B * nL * Hq > (1LL << 31) / 2) return HD_ERR_UNSUPPORTED;
@@ -234,7 +234,10 @@ hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float*
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  if (use_mma_kernels()) return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  // head dim 256 (no room for its O and S accumulators beside a second query tile in
+  // TMEM) runs on the mma.sync kernel
+  if (use_mma_kernels() || Dh == 256)
+    return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
   return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
 }
 
@@ -292,7 +295,8 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  // head dim 128 runs on the tcgen05 kernel; head dim 64 on the mma.sync kernel
+  // head dim 128 runs on the tcgen05 kernel; head dims 64 and 256 on the mma.sync kernel
+  // (at 256 in two launches, one per half of the dK / dV / dQ columns)
   if (Dh == 128 && !use_mma_kernels())
     return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
                                                      scale, dev_status, stream));
@@ -390,7 +394,8 @@ hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, 
   SfaGeom g;
   hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
-  if (use_mma_kernels()) return HD_ERR_UNSUPPORTED;  // the mma.sync kernels have no final-stream geometry
+  // the mma.sync kernels (HDSFA_KERNELS=mma, head dim 256) have no final-stream geometry
+  if (use_mma_kernels() || Dh == 256) return HD_ERR_UNSUPPORTED;
   return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, resolve_scale(softmax_scale, Dh), dev_status,
                                               stream));
 }

@@ -113,7 +113,12 @@ cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* ls
   const long long warps = (rows + rpw - 1) / rpw;
   const unsigned blocks = (unsigned)((warps * 32 + 255) / 256);
   const bf16 *ob = (const bf16*)o, *db = (const bf16*)dout;
-  if (Dh == 64) {
+  if (Dh == 256) {
+    if (zero)
+      sfa_bwd_prep_kernel<256, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+    else
+      sfa_bwd_prep_kernel<256, false><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+  } else if (Dh == 64) {
     if (zero)
       sfa_bwd_prep_kernel<64, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
     else

@@ -40,6 +40,7 @@ struct MmaBwdArgs {
   SfaGeom g;
   float scale;
   float scale_log2;
+  int d0;  // first head-dim column of the dK / dV / dQ slice this launch writes
 };
 
 // rows [r0, r0 + ROWS) of a [*][DH] row set (row stride rstride elements) -> swizzled smem.
@@ -86,7 +87,10 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
   load_rows<DH, BN>(sV, vb, kv_rs, n_lo * BN, G.Lv, tid);
   cp_async_commit();
 
-  uint32_t qf[DH / 16][4];
+  // Q fragments stay in registers up to head dim 128; at 256 the O accumulator needs
+  // those registers and the fragments are reloaded from shared memory per key tile.
+  constexpr bool kHoldQ = DH <= 128;
+  uint32_t qf[kHoldQ ? DH / 16 : 1][4];
   float oacc[DH / 8][4];
 #pragma unroll
   for (int i = 0; i < DH / 8; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
@@ -98,9 +102,9 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
     const int buf = (nt_i - n_lo) & 1;
     cp_async_wait<0>();
     __syncthreads();
-    if (nt_i == n_lo) {
+    if (kHoldQ && nt_i == n_lo) {
 #pragma unroll
-      for (int kk = 0; kk < DH / 16; ++kk)
+      for (int kk = 0; kk < (kHoldQ ? DH / 16 : 0); ++kk)
         ldsm_x4(smem_u32(sQ + swz<DH>(warp * 16 + (lane & 15), kk * 16 + (lane >> 4) * 8)),
                 qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
     }
@@ -118,14 +122,24 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
     for (int i = 0; i < BN / 8; ++i) sacc[i][0] = sacc[i][1] = sacc[i][2] = sacc[i][3] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < DH / 16; ++kk) {
+      uint32_t qr[4];
+      if (kHoldQ) {
+        qr[0] = qf[kHoldQ ? kk : 0][0];
+        qr[1] = qf[kHoldQ ? kk : 0][1];
+        qr[2] = qf[kHoldQ ? kk : 0][2];
+        qr[3] = qf[kHoldQ ? kk : 0][3];
+      } else {
+        ldsm_x4(smem_u32(sQ + swz<DH>(warp * 16 + (lane & 15), kk * 16 + (lane >> 4) * 8)), qr[0], qr[1], qr[2],
+                qr[3]);
+      }
 #pragma unroll
       for (int np = 0; np < BN / 16; ++np) {
         uint32_t b0, b1, b2, b3;
         ldsm_x4(smem_u32(cK + swz<DH>(np * 16 + (lane & 7) + (lane >> 4) * 8,
                                       kk * 16 + ((lane >> 3) & 1) * 8)),
                 b0, b1, b2, b3);
-        mma_bf16_16816(sacc[2 * np], qf[kk], b0, b1);
-        mma_bf16_16816(sacc[2 * np + 1], qf[kk], b2, b3);
+        mma_bf16_16816(sacc[2 * np], qr, b0, b1);
+        mma_bf16_16816(sacc[2 * np + 1], qr, b2, b3);
       }
     }
     const bool need_mask = (nt_i == n_hi) || G.window > 0;
@@ -225,7 +239,10 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
 // registers while looping over the group's query heads and the query tiles that
 // can see tile j; dQ contributions go to the fp32 accumulator with atomics.
 // Warp w owns key rows [16w, 16w + 16) of the tile for S^T, dP^T, dK, dV.
-template <int DH>
+// DO: the head-dim columns of dK, dV, dQ one launch accumulates (starting at a.d0);
+// S^T and dP^T always take the full head dim.  DO = DH in one launch, or two launches
+// of DO = DH / 2 at head dim 256 (whose dK and dV would not fit the registers at once).
+template <int DH, int DO>
 __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem_raw[];
   bf16* sK = reinterpret_cast<bf16*>(smem_raw);  // [BN][DH]
@@ -279,9 +296,9 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
     sD[tid] = dl;
   }
 
-  float dK[DH / 8][4], dV[DH / 8][4];
+  float dK[DO / 8][4], dV[DO / 8][4];
 #pragma unroll
-  for (int i = 0; i < DH / 8; ++i)
+  for (int i = 0; i < DO / 8; ++i)
 #pragma unroll
     for (int e = 0; e < 4; ++e) dK[i][e] = dV[i][e] = 0.f;
 
@@ -360,8 +377,8 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
         da[3] = pack_bf16(dpacc[2 * kk + 1][2], dpacc[2 * kk + 1][3]);
         const int qrow = half * 32 + kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
-        for (int dp = 0; dp < DH / 16; ++dp) {
-          const int dcol = dp * 16 + (lane >> 4) * 8;
+        for (int dp = 0; dp < DO / 16; ++dp) {
+          const int dcol = a.d0 + dp * 16 + (lane >> 4) * 8;
           uint32_t b0, b1, b2, b3;
           ldsm_x4_t(smem_u32(cdO + swz<DH>(qrow, dcol)), b0, b1, b2, b3);
           mma_bf16_16816(dV[2 * dp], pa, b0, b1);
@@ -386,9 +403,9 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
       const int qa = m0 + warp * 16 + g4;
 #pragma unroll
       for (int dh = 0; dh < 2; ++dh) {
-        float qacc[DH / 16][4];
+        float qacc[DO / 16][4];
 #pragma unroll
-        for (int i = 0; i < DH / 16; ++i) qacc[i][0] = qacc[i][1] = qacc[i][2] = qacc[i][3] = 0.f;
+        for (int i = 0; i < DO / 16; ++i) qacc[i][0] = qacc[i][1] = qacc[i][2] = qacc[i][3] = 0.f;
 #pragma unroll
         for (int kk = 0; kk < BN / 16; ++kk) {
           uint32_t aa[4];
@@ -396,18 +413,18 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
                                            warp * 16 + ((lane >> 3) & 1) * 8)),
                     aa[0], aa[1], aa[2], aa[3]);
 #pragma unroll
-          for (int dp = 0; dp < DH / 32; ++dp) {
+          for (int dp = 0; dp < DO / 32; ++dp) {
             uint32_t b0, b1, b2, b3;
             ldsm_x4_t(smem_u32(sK + swz<DH>(kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8,
-                                            dh * (DH / 2) + dp * 16 + (lane >> 4) * 8)),
+                                            a.d0 + dh * (DO / 2) + dp * 16 + (lane >> 4) * 8)),
                       b0, b1, b2, b3);
             mma_bf16_16816(qacc[2 * dp], aa, b0, b1);
             mma_bf16_16816(qacc[2 * dp + 1], aa, b2, b3);
           }
         }
 #pragma unroll
-        for (int i = 0; i < DH / 16; ++i) {
-          const int col = dh * (DH / 2) + i * 8 + 2 * t4;
+        for (int i = 0; i < DO / 16; ++i) {
+          const int col = a.d0 + dh * (DO / 2) + i * 8 + 2 * t4;
           if (qa < G.Lv)
             atomicAdd(reinterpret_cast<float2*>(dqb + (long long)qa * q_rs + col),
                       make_float2(qacc[i][0], qacc[i][1]));
@@ -428,8 +445,8 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   bf16* dvb = a.dv + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
   const int kr = n0 + warp * 16 + g4;
 #pragma unroll
-  for (int i = 0; i < DH / 8; ++i) {
-    const int col = i * 8 + 2 * t4;
+  for (int i = 0; i < DO / 8; ++i) {
+    const int col = a.d0 + i * 8 + 2 * t4;
     if (kr < G.Lv) {
       *reinterpret_cast<uint32_t*>(dkb + (long long)kr * kv_rs + col) =
           pack_bf16(dK[i][0] * a.scale, dK[i][1] * a.scale);
@@ -459,7 +476,25 @@ static cudaError_t fwd_impl(const MmaFwdArgs& a, cudaStream_t st) {
 cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
                                const SfaGeom& g, int Dh, float scale, cudaStream_t st) {
   MmaFwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (bf16*)o, lse, g, scale * kLog2e};
-  return Dh == 64 ? fwd_impl<64>(a, st) : fwd_impl<128>(a, st);
+  if (Dh == 64) return fwd_impl<64>(a, st);
+  if (Dh == 256) return fwd_impl<256>(a, st);
+  return fwd_impl<128>(a, st);
+}
+
+template <int DH, int DO>
+static cudaError_t bwd_impl(MmaBwdArgs a, cudaStream_t st) {
+  const SfaGeom& g = a.g;
+  const int smem = (2 * BN * DH + 4 * BM * DH + BN * BM) * (int)sizeof(bf16) + 4 * BM * (int)sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<DH, DO>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.ns, g.B);
+  for (int d0 = 0; d0 < DH; d0 += DO) {  // one launch per output slice
+    a.d0 = d0;
+    sfa_bwd_mma_kernel<DH, DO><<<grid, NT, smem, st>>>(a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const void* dout,
@@ -467,24 +502,10 @@ cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v,
                                     float* dq_ws, const SfaGeom& g, int Dh, float scale,
                                     cudaStream_t st) {
   MmaBwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)dout, lse2_ws, delta_ws,
-               dq_ws, (bf16*)dk, (bf16*)dv, g, scale, scale * kLog2e};
-  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.ns, g.B);
-  auto smem_of = [](int dh) {
-    return (2 * BN * dh + 4 * BM * dh + BN * BM) * (int)sizeof(bf16) + 4 * BM * (int)sizeof(float);
-  };
-  cudaError_t e;
-  if (Dh == 64) {
-    const int smem = smem_of(64);
-    e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    sfa_bwd_mma_kernel<64><<<grid, NT, smem, st>>>(a);
-  } else {
-    const int smem = smem_of(128);
-    e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    sfa_bwd_mma_kernel<128><<<grid, NT, smem, st>>>(a);
-  }
-  return cudaGetLastError();
+               dq_ws, (bf16*)dk, (bf16*)dv, g, scale, scale * kLog2e, 0};
+  if (Dh == 64) return bwd_impl<64, 64>(a, st);
+  if (Dh == 256) return bwd_impl<256, 128>(a, st);
+  return bwd_impl<128, 128>(a, st);
 }
 
 }  // namespace hdsfa

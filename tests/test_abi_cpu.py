@@ -62,7 +62,7 @@ def test_fwd_validation(lib):
     assert _fwd(lib, ptr=FAKE + 8) == 1         # misaligned
     assert _fwd(lib, ptr=0) == 1                # null
     assert _fwd(lib, Dh=96) == 2                # unsupported head dim
-    assert _fwd(lib, Dh=256) == 2
+    assert _fwd(lib, Dh=32) == 2
 
 
 def test_bwd_workspace_size(lib):
@@ -178,6 +178,8 @@ def test_final_stream_validation(lib):
     P, Z, F = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_float
     assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 128, 1) > 0
     assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 64, 1) == 0    # backward: head dim 128 only
+    assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 64, 4, 8, 2, 256, F(0.0), 1, 0,
+                             None, None) == 2                                # no head dim 256 here
     assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE + 4), 1, 64, 4, 8, 2, 128, F(0.0), 1, 0,
                              None, None) == 1
     assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 64, 4, 8, 3, 128, F(0.0), 1, 0,

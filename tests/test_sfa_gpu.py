@@ -64,6 +64,14 @@ def test_wide_gqa_groups(mode, window):
     _full_case(AttnShape(2, 150, 4, 6, 2, 128), mode, seed=22, window=window)
 
 
+@pytest.mark.parametrize("mode,window", [(WITHIN, 0), (CROSS, 0), (LOCAL, 40)])
+def test_head_dim_256(mode, window):
+    # head dim 256 (the paper's 80B configuration, 24 query over 2 K/V heads, Table 6) on
+    # the mma.sync kernels: the backward in two launches over halves of the head dim
+    _full_case(AttnShape(1, 70, 4, 24, 2, 256), mode, seed=31, window=window)
+    _full_case(AttnShape(2, 33, 2, 4, 4, 256), mode, seed=32, window=window)
+
+
 @pytest.mark.parametrize("window", [1, 50, 200])
 def test_local_window(window):
     _full_case(AttnShape(1, 96, 4, 4, 2, 128), LOCAL, seed=5, window=window)
