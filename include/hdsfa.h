@@ -204,8 +204,8 @@ hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int
  *   lse            : float32 [B][Hq][L], natural log (written by sfa_fwd_final)
  * dk, dv are fully overwritten (zero for keys no final-stream query sees).
  * workspace: >= sfa_bwd_final_workspace_bytes(...) bytes, 256-byte aligned.
- * sfa_fwd_final takes Dh in {64, 128}; sfa_bwd_final Dh = 128 (HD_ERR_UNSUPPORTED
- * otherwise); both run on the tcgen05 kernels (HDSFA_KERNELS=mma: HD_ERR_UNSUPPORTED).
+ * Dh in {64, 128, 256}: head dim 128 runs on the tcgen05 kernels, 64 (backward) and 256
+ * on the mma.sync kernels, as in sfa_fwd / sfa_bwd.
  */
 hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
                           int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,

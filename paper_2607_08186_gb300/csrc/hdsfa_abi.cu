@@ -394,15 +394,15 @@ hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, 
   SfaGeom g;
   hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
-  // the mma.sync kernels (HDSFA_KERNELS=mma, head dim 256) have no final-stream geometry
-  if (use_mma_kernels() || Dh == 256) return HD_ERR_UNSUPPORTED;
-  return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, resolve_scale(softmax_scale, Dh), dev_status,
-                                              stream));
+  const float scale = resolve_scale(softmax_scale, Dh);
+  if (use_mma_kernels() || Dh == 256)  // head dim 256: the mma.sync kernel, as in sfa_fwd
+    return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
 }
 
 size_t sfa_bwd_final_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode) {
   SfaGeom g;
-  if (Dh != 128 || make_final_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g) != HD_OK) return 0;
+  if (make_final_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g) != HD_OK) return 0;
   return ws_bytes(g, Dh);
 }
 
@@ -416,7 +416,7 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
   SfaGeom g;
   hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
-  if (Dh != 128 || use_mma_kernels()) return HD_ERR_UNSUPPORTED;  // the tcgen05 backward is head dim 128
+
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
@@ -428,8 +428,13 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
     e = cudaMemsetAsync(dk, 0, bytes, stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(dv, 0, bytes, stream);
   }
-  if (e == cudaSuccess)
-    e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status, stream);
+  if (e == cudaSuccess) {
+    if (Dh == 128 && !use_mma_kernels())
+      e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status,
+                                        stream);
+    else  // head dims 64 and 256 on the mma.sync kernel
+      e = hdsfa::launch_sfa_bwd_main_mma(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh, scale, stream);
+  }
   if (e == cudaSuccess) e = hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, gq, Dh, scale, stream);
   return cuda_status(e);
 }

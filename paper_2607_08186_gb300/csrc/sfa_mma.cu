@@ -5,7 +5,8 @@
 // Each CTA works on one virtual causal problem (see SfaGeom): WITHIN mode gives
 // one problem per stream (rows p = r*n + s, Eq. 4), so a query tile visits only
 // its own stream's key tiles; CROSS gives one causal problem over nL positions
-// (Fig. 2a); LOCAL adds the window bound (Fig. 2b).  Key tiles beyond the causal
+// (Fig. 2a); LOCAL adds the window bound (Fig. 2b); a final-stream problem maps
+// query row r to key row r*qstep + qoff.  Key tiles beyond the causal
 // diagonal (or before the window) are never visited; only tiles that straddle a
 // mask edge are masked in registers.
 #include "common.cuh"
@@ -57,8 +58,10 @@ HD_DEVINLINE void load_rows(bf16* s, const bf16* base, long long rstride, int r0
   }
 }
 
-HD_DEVINLINE bool visible(int r, int c, int Lv, int window) {
-  return c <= r && c < Lv && (window <= 0 || r - c < window);
+// Key row c visible from the query at key row rq (query row r sits at key row
+// r*qstep + qoff of its problem: r itself unless it is a final-stream problem).
+HD_DEVINLINE bool visible(int rq, int c, int Lv, int window) {
+  return c <= rq && c < Lv && (window <= 0 || rq - c < window);
 }
 
 // ----------------------------------------------------------------- forward
@@ -70,19 +73,21 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
   bf16* sV = sK + 2 * BN * DH;                    // [2][BN][DH]
   const SfaGeom G = a.g;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int ntile = (G.Lv + BM - 1) / BM;
+  const int ntile = (G.Lq + BM - 1) / BM;
   const int mt = ntile - 1 - (int)blockIdx.x;  // longest rows first
   const int m0 = mt * BM;
-  const int h = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
+  const int h = blockIdx.y / G.q_ns, s = blockIdx.y % G.q_ns, b = blockIdx.z;
+  const int sk = s + G.kv_s0;  // stream of the key problem
   const int kvh = h / (G.Hq / G.Hkv);
-  const long long q_rs = (long long)G.rs * G.Hq * DH, kv_rs = (long long)G.rs * G.Hkv * DH;
-  const bf16* qb = a.q + (((long long)b * G.nL + s) * G.Hq + h) * DH;
-  const bf16* kb = a.k + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
-  const bf16* vb = a.v + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
-  const int n_lo = G.window > 0 ? max(0, m0 - G.window + 1) / BN : 0;
-  const int n_hi = mt;  // BM == BN: the diagonal tile
+  const long long q_rs = (long long)G.q_rs * G.Hq * DH, kv_rs = (long long)G.rs * G.Hkv * DH;
+  const bf16* qb = a.q + (((long long)b * G.q_nL + s) * G.Hq + h) * DH;
+  const bf16* kb = a.k + (((long long)b * G.nL + sk) * G.Hkv + kvh) * DH;
+  const bf16* vb = a.v + (((long long)b * G.nL + sk) * G.Hkv + kvh) * DH;
+  const int rq_first = m0 * G.qstep + G.qoff, rq_last = (min(m0 + BM, G.Lq) - 1) * G.qstep + G.qoff;
+  const int n_lo = G.window > 0 ? max(0, rq_first - G.window + 1) / BN : 0;
+  const int n_hi = min(rq_last / BN, (G.Lv - 1) / BN);
 
-  load_rows<DH, BM>(sQ, qb, q_rs, m0, G.Lv, tid);
+  load_rows<DH, BM>(sQ, qb, q_rs, m0, G.Lq, tid);
   load_rows<DH, BN>(sK, kb, kv_rs, n_lo * BN, G.Lv, tid);
   load_rows<DH, BN>(sV, vb, kv_rs, n_lo * BN, G.Lv, tid);
   cp_async_commit();
@@ -142,7 +147,8 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
         mma_bf16_16816(sacc[2 * np + 1], qr, b2, b3);
       }
     }
-    const bool need_mask = (nt_i == n_hi) || G.window > 0;
+    // tiles with a key past the first query's key row, under a window, or ragged
+    const bool need_mask = (nt_i + 1) * BN - 1 > rq_first || G.window > 0 || (nt_i + 1) * BN > G.Lv;
     float tmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
     for (int i = 0; i < BN / 8; ++i) {
@@ -151,7 +157,7 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
         float x = sacc[i][e] * a.scale_log2;
         if (need_mask) {
           const int r = r_lo + (e >> 1) * 8, c = n0 + i * 8 + 2 * t4 + (e & 1);
-          if (!visible(r, c, G.Lv, G.window)) x = -INFINITY;
+          if (!visible(r * G.qstep + G.qoff, c, G.Lv, G.window)) x = -INFINITY;
         }
         sacc[i][e] = x;
         tmax[e >> 1] = fmaxf(tmax[e >> 1], x);
@@ -219,16 +225,16 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
     *reinterpret_cast<uint32_t*>(sQ + swz<DH>(row + 8, col)) = pack_bf16(oacc[i][2] * inv1, oacc[i][3] * inv1);
   }
   if (t4 == 0) {
-    float* lrow = a.lse + ((long long)b * G.Hq + h) * G.nL + s;
-    if (r_lo < G.Lv) lrow[(long long)r_lo * G.rs] = (mx[0] + log2f(lsum[0])) * kLn2;
-    if (r_lo + 8 < G.Lv) lrow[(long long)(r_lo + 8) * G.rs] = (mx[1] + log2f(lsum[1])) * kLn2;
+    float* lrow = a.lse + ((long long)b * G.Hq + h) * G.q_nL + s;
+    if (r_lo < G.Lq) lrow[(long long)r_lo * G.q_rs] = (mx[0] + log2f(lsum[0])) * kLn2;
+    if (r_lo + 8 < G.Lq) lrow[(long long)(r_lo + 8) * G.q_rs] = (mx[1] + log2f(lsum[1])) * kLn2;
   }
   __syncthreads();
-  bf16* ob = a.o + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+  bf16* ob = a.o + (((long long)b * G.q_nL + s) * G.Hq + h) * DH;
   constexpr int CPR = DH / 8;
   for (int i = tid; i < BM * CPR; i += NT) {
     const int r = i / CPR, c = i % CPR;
-    if (m0 + r < G.Lv)
+    if (m0 + r < G.Lq)
       *reinterpret_cast<uint4*>(ob + (long long)(m0 + r) * q_rs + c * 8) =
           *reinterpret_cast<const uint4*>(sQ + swz<DH>(r, c * 8));
   }
@@ -256,40 +262,44 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   const SfaGeom G = a.g;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g4 = lane >> 2, t4 = lane & 3;
-  const int ntile = (G.Lv + BM - 1) / BM;
+  const int ntile = (G.Lq + BM - 1) / BM;
   const int j = blockIdx.x;  // key tile; tile 0 sees the most query tiles, so it starts first
   const int n0 = j * BN;
-  const int kvh = blockIdx.y / G.ns, s = blockIdx.y % G.ns, b = blockIdx.z;
+  const int kvh = blockIdx.y / G.q_ns, s = blockIdx.y % G.q_ns, b = blockIdx.z;
+  const int sk = s + G.kv_s0;  // stream of the key problem
   const int grp = G.Hq / G.Hkv;
+  // query tiles that can see a key of this tile: query row r stands at key row
+  // r*qstep + qoff >= n0, and under a window r*qstep + qoff < n0 + BN - 1 + window
+  const int mi_lo = (n0 <= G.qoff ? 0 : (n0 - G.qoff + G.qstep - 1) / G.qstep) / BM;
   int mi_hi = ntile - 1;
-  if (G.window > 0) mi_hi = min(mi_hi, (n0 + BN - 1 + G.window - 1) / BM);
-  const int nq = mi_hi - j + 1;
-  const int total = grp * nq;
-  const long long q_rs = (long long)G.rs * G.Hq * DH, kv_rs = (long long)G.rs * G.Hkv * DH;
-  const bf16* kb = a.k + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
-  const bf16* vb = a.v + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  if (G.window > 0) mi_hi = min(mi_hi, ((n0 + BN - 2 + G.window - G.qoff) / G.qstep) / BM);
+  const int nq = mi_hi - mi_lo + 1;
+  const int total = grp * max(nq, 0);
+  const long long q_rs = (long long)G.q_rs * G.Hq * DH, kv_rs = (long long)G.rs * G.Hkv * DH;
+  const bf16* kb = a.k + (((long long)b * G.nL + sk) * G.Hkv + kvh) * DH;
+  const bf16* vb = a.v + (((long long)b * G.nL + sk) * G.Hkv + kvh) * DH;
 
   auto q_base = [&](const bf16* t, int h) {
-    return t + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+    return t + (((long long)b * G.q_nL + s) * G.Hq + h) * DH;
   };
-  const int Lvp = row_terms_pitch(G.Lv);
+  const int Lqp = row_terms_pitch(G.Lq);
   auto row_terms = [&](int it, int r, float& l2, float& dl) {
-    const int h = kvh * grp + it / nq, m0 = (j + it % nq) * BM;
-    const long long idx = (((long long)b * G.Hq + h) * G.ns + s) * Lvp + m0 + r;
-    const bool ok = m0 + r < G.Lv;
+    const int h = kvh * grp + it / nq, m0 = (mi_lo + it % nq) * BM;
+    const long long idx = (((long long)b * G.Hq + h) * G.q_ns + s) * Lqp + m0 + r;
+    const bool ok = m0 + r < G.Lq;
     l2 = ok ? a.lse2[idx] : 0.f;
     dl = ok ? a.delta[idx] : 0.f;
   };
 
   load_rows<DH, BN>(sK, kb, kv_rs, n0, G.Lv, tid);
   load_rows<DH, BN>(sV, vb, kv_rs, n0, G.Lv, tid);
-  {
+  if (total > 0) {
     const int h = kvh * grp;
-    load_rows<DH, BM>(sQ, q_base(a.q, h), q_rs, j * BM, G.Lv, tid);
-    load_rows<DH, BM>(sdO, q_base(a.dout, h), q_rs, j * BM, G.Lv, tid);
+    load_rows<DH, BM>(sQ, q_base(a.q, h), q_rs, mi_lo * BM, G.Lq, tid);
+    load_rows<DH, BM>(sdO, q_base(a.dout, h), q_rs, mi_lo * BM, G.Lq, tid);
   }
   cp_async_commit();
-  if (tid < BM) {
+  if (tid < BM && total > 0) {
     float l2, dl;
     row_terms(0, tid, l2, dl);
     sL[tid] = l2;
@@ -309,14 +319,14 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
     const bool has_next = it + 1 < total;
     float nl2 = 0.f, ndl = 0.f;
     if (has_next) {
-      const int h1 = kvh * grp + (it + 1) / nq, m1 = (j + (it + 1) % nq) * BM;
-      load_rows<DH, BM>(sQ + (buf ^ 1) * BM * DH, q_base(a.q, h1), q_rs, m1, G.Lv, tid);
-      load_rows<DH, BM>(sdO + (buf ^ 1) * BM * DH, q_base(a.dout, h1), q_rs, m1, G.Lv, tid);
+      const int h1 = kvh * grp + (it + 1) / nq, m1 = (mi_lo + (it + 1) % nq) * BM;
+      load_rows<DH, BM>(sQ + (buf ^ 1) * BM * DH, q_base(a.q, h1), q_rs, m1, G.Lq, tid);
+      load_rows<DH, BM>(sdO + (buf ^ 1) * BM * DH, q_base(a.dout, h1), q_rs, m1, G.Lq, tid);
       cp_async_commit();
       if (tid < BM) row_terms(it + 1, tid, nl2, ndl);
     }
     const int h = kvh * grp + it / nq;
-    const int m0 = (j + it % nq) * BM;
+    const int m0 = (mi_lo + it % nq) * BM;
     const bf16* cQ = sQ + buf * BM * DH;
     const bf16* cdO = sdO + buf * BM * DH;
     const float* cL = sL + buf * BM;
@@ -358,7 +368,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
           const int ql = half * 32 + i * 8 + 2 * t4 + (e & 1);
           const int qr = m0 + ql;
           float p = 0.f;
-          if (visible(qr, kr, G.Lv, G.window) && qr < G.Lv)
+          if (qr < G.Lq && visible(qr * G.qstep + G.qoff, kr, G.Lv, G.window))
             p = exp2f(fmaf(sacc[i][e], a.scale_log2, cL[ql]));
           sacc[i][e] = p;
           dpacc[i][e] = p * (dpacc[i][e] + cD[ql]);
@@ -399,7 +409,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
     __syncthreads();
     // dQ[q rows of warp] += dS K  (unscaled; the post kernel applies the scale)
     {
-      float* dqb = a.dq_acc + (((long long)b * G.nL + s) * G.Hq + h) * DH;
+      float* dqb = a.dq_acc + (((long long)b * G.q_nL + s) * G.Hq + h) * DH;
       const int qa = m0 + warp * 16 + g4;
 #pragma unroll
       for (int dh = 0; dh < 2; ++dh) {
@@ -425,10 +435,10 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
 #pragma unroll
         for (int i = 0; i < DO / 16; ++i) {
           const int col = a.d0 + dh * (DO / 2) + i * 8 + 2 * t4;
-          if (qa < G.Lv)
+          if (qa < G.Lq)
             atomicAdd(reinterpret_cast<float2*>(dqb + (long long)qa * q_rs + col),
                       make_float2(qacc[i][0], qacc[i][1]));
-          if (qa + 8 < G.Lv)
+          if (qa + 8 < G.Lq)
             atomicAdd(reinterpret_cast<float2*>(dqb + (long long)(qa + 8) * q_rs + col),
                       make_float2(qacc[i][2], qacc[i][3]));
         }
@@ -440,9 +450,10 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
     }
   }
 
+  cp_async_wait<0>();  // a key tile that no query sees still loaded K and V
   // epilogue: dK *= scale, write dK and dV rows of this key tile
-  bf16* dkb = a.dk + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
-  bf16* dvb = a.dv + (((long long)b * G.nL + s) * G.Hkv + kvh) * DH;
+  bf16* dkb = a.dk + (((long long)b * G.nL + sk) * G.Hkv + kvh) * DH;
+  bf16* dvb = a.dv + (((long long)b * G.nL + sk) * G.Hkv + kvh) * DH;
   const int kr = n0 + warp * 16 + g4;
 #pragma unroll
   for (int i = 0; i < DO / 8; ++i) {
@@ -468,7 +479,7 @@ static cudaError_t fwd_impl(const MmaFwdArgs& a, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(sfa_fwd_mma_kernel<DH>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((a.g.Lv + BM - 1) / BM, a.g.Hq * a.g.ns, a.g.B);
+  dim3 grid((a.g.Lq + BM - 1) / BM, a.g.Hq * a.g.q_ns, a.g.B);
   sfa_fwd_mma_kernel<DH><<<grid, NT, smem, st>>>(a);
   return cudaGetLastError();
 }
@@ -487,7 +498,7 @@ static cudaError_t bwd_impl(MmaBwdArgs a, cudaStream_t st) {
   const int smem = (2 * BN * DH + 4 * BM * DH + BN * BM) * (int)sizeof(bf16) + 4 * BM * (int)sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<DH, DO>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.ns, g.B);
+  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.q_ns, g.B);
   for (int d0 = 0; d0 < DH; d0 += DO) {  // one launch per output slice
     a.d0 = d0;
     sfa_bwd_mma_kernel<DH, DO><<<grid, NT, smem, st>>>(a);

@@ -177,9 +177,8 @@ def test_kv_append_validation(lib):
 def test_final_stream_validation(lib):
     P, Z, F = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_float
     assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 128, 1) > 0
-    assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 64, 1) == 0    # backward: head dim 128 only
-    assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 64, 4, 8, 2, 256, F(0.0), 1, 0,
-                             None, None) == 2                                # no head dim 256 here
+    assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 256, 1) > 0
+    assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 80, 1) == 0     # unsupported head dim
     assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE + 4), 1, 64, 4, 8, 2, 128, F(0.0), 1, 0,
                              None, None) == 1
     assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 64, 4, 8, 3, 128, F(0.0), 1, 0,
@@ -187,5 +186,6 @@ def test_final_stream_validation(lib):
     assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 64, 4, 8, 2, 96, F(0.0), 1, 0,
                              None, None) == 2
     a = [P(FAKE)] * 9
-    assert lib.sfa_bwd_final(*a, 1, 64, 4, 8, 2, 64, F(0.0), 1, 0, P(FAKE), Z(1 << 30), None, None) == 2
+    assert lib.sfa_bwd_final(*a, 1, 64, 4, 8, 2, 96, F(0.0), 1, 0, P(FAKE), Z(1 << 30), None, None) == 2
     assert lib.sfa_bwd_final(*a, 1, 64, 4, 8, 2, 128, F(0.0), 1, 0, P(FAKE), Z(16), None, None) == 4
+    assert lib.sfa_bwd_final(*a, 1, 64, 4, 8, 2, 256, F(0.0), 1, 0, P(FAKE), Z(16), None, None) == 4

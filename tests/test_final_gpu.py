@@ -77,6 +77,20 @@ def test_fwd_bwd_shapes(mode, w, B, L, n, Hq, Hkv):
             assert torch.count_nonzero(got["dk"][:, s::n]) == 0 and torch.count_nonzero(got["dv"][:, s::n]) == 0
 
 
+@pytest.mark.parametrize("mode,w", [(WITHIN, 0), (CROSS, 0), (LOCAL, 9)])
+@pytest.mark.parametrize("B,L,n,Hq,Hkv,Dh", [(1, 70, 4, 24, 2, 256), (2, 40, 3, 4, 4, 256), (1, 90, 2, 4, 2, 64)])
+def test_mma_kernels_fwd_bwd(mode, w, B, L, n, Hq, Hkv, Dh):
+    # head dim 256 (the 80B final-stream-only layers: 24 over 2 heads, Table 6) and head
+    # dim 64 run the final-stream geometry on the mma.sync kernels
+    q, k, v, do = _inputs(B, L, n, Hq, Hkv, Dh, L + Dh)
+    got = _gpu(q, k, v, do, mode, w)
+    o_r, lse_r = oracle.sfa_fwd_final(q, k, v, n, mode, window=w)
+    assert float((got["o"].double() - o_r).abs().max()) <= 2e-2
+    assert float((got["lse"].double() - lse_r).abs().max()) <= 1e-3
+    for name, r in zip(("dq", "dk", "dv"), oracle.sfa_bwd_final(q, k, v, do, n, mode, window=w)):
+        assert _rel(got[name], r) <= 1e-2, (name, _rel(got[name], r))
+
+
 @pytest.mark.parametrize("mode", [WITHIN, CROSS])
 def test_fwd_head_dim_64(mode):
     q, k, v, do = _inputs(2, 150, 4, 4, 2, 64, 3)
