@@ -95,6 +95,9 @@ struct Params {
 };
 
 
+// WIN: a windowed (LOCAL) problem, whose pre-fill masks only tiles that reach the
+// window edge; the other modes keep a separate instantiation.
+template <bool WIN>
 __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant__ Params P) {
   extern __shared__ uint8_t smem_raw[];
   {
@@ -471,7 +474,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         w[4 * i + 2] = __float_as_uint(x.z * inv_c2);
         w[4 * i + 3] = __float_as_uint(x.w * inv_c2);
       }
-      if ((qm * G.qstep + G.qoff < n0 + BK) || G.window > 0 || (n0 + BK > G.Lv) || (qm + BQ > G.Lq)) {
+      // masked where a pair can fall outside: the diagonal band, (LOCAL) the last query's
+      // window edge at or above the tile's first key, ragged tiles
+      const bool win_edge =
+          WIN ? (qm + BQ - 1) * G.qstep + G.qoff - G.window >= n0 : G.window > 0;
+      if ((qm * G.qstep + G.qoff < n0 + BK) || win_edge || (n0 + BK > G.Lv) || (qm + BQ > G.Lq)) {
         // key row kr sees the queries q in [vis_lo, vis_hi): q*qstep + qoff >= kr
         // (causal), q < Lq, and for LOCAL q*qstep + qoff < kr + window (an empty range
         // when kr itself is past Lv)
@@ -617,10 +624,11 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   p.scale_log2 = scale * 1.4426950408889634f;
   p.status = status;
   const int smem = kSmemBytes;
-  cudaError_t e = cudaFuncSetAttribute(bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  auto kern = g.window > 0 ? bwd_kernel<true> : bwd_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.q_ns * g.B);
-  bwd_kernel<<<grid, NTHREADS, smem, st>>>(p);
+  kern<<<grid, NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }
 

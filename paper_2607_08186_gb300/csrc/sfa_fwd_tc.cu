@@ -218,6 +218,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     const int r = m0 + g * BM + row;
     const int rq = r * G.qstep + G.qoff;                      // its key row
     const int rq0 = (m0 + g * BM) * G.qstep + G.qoff;         // key row of the tile's first query
+    // key row of its last query (a key tile above rq1 - window is inside every row's window)
+    const int rq1 = (min(m0 + g * BM + BM, G.Lq) - 1) * G.qstep + G.qoff;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     const uint32_t tS = tl + g * 128, tO = tl + 256 + g * DH;
     const float c2 = P.scale_log2;
@@ -235,9 +237,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
       for (int c = 0; c < BN / 32; ++c) tmem_ld32(tS + c * 32, reinterpret_cast<uint32_t*>(x) + c * 32);
       tmem_ld_wait();
-      // tiles holding a key past the first query's key row (the diagonal band), any tile
-      // under a window, and the ragged last tile
-      const bool need_mask = (j + 1) * BN - 1 > rq0 || G.window > 0 || (j + 1) * BN > G.Lv;
+      // tiles holding a key past the first query's key row (the diagonal band), a key at
+      // or below the last query's window edge, and the ragged last tile
+      const bool need_mask = (j + 1) * BN - 1 > rq0 || (G.window > 0 && j * BN <= rq1 - G.window) ||
+                             (j + 1) * BN > G.Lv;
       if (need_mask) {
 #pragma unroll
         for (int e = 0; e < BN; ++e)
