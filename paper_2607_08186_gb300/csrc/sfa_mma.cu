@@ -147,8 +147,10 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
         mma_bf16_16816(sacc[2 * np + 1], qr, b2, b3);
       }
     }
-    // tiles with a key past the first query's key row, under a window, or ragged
-    const bool need_mask = (nt_i + 1) * BN - 1 > rq_first || G.window > 0 || (nt_i + 1) * BN > G.Lv;
+    // tiles with a key past the first query's key row, a key at or below the last
+    // query's window edge, or ragged
+    const bool need_mask = (nt_i + 1) * BN - 1 > rq_first || (G.window > 0 && nt_i * BN <= rq_last - G.window) ||
+                           (nt_i + 1) * BN > G.Lv;
     float tmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
     for (int i = 0; i < BN / 8; ++i) {
