@@ -10,11 +10,13 @@ this module compiles it with gcc on first use and marshals torch/numpy arrays
 to it.  Every function takes float tensors of any dtype and upcasts them to
 fp64 exactly (bf16 -> fp64 is exact).
 
-Citations (Hidden Decoding paper): Eq. 1 (expansion), Eq. 3 (token / stream
+Citations (Hidden Decoding paper): Eq. 1 (expansion, and its adjoint into the n
+tables), Eq. 2 (the final-stream positions the loss reads), Eq. 3 (token / stream
 index), Eq. 4 (intra-stream mask), Fig. 2 (full and local cross-stream masks),
 Sec. 2 "Setup" (standard causal softmax attention, grouped K/V heads per
-Table 6).  The backward is the derivative of that forward (the paper does not
-write it out).
+Table 6), Sec. 3.1 (final-stream-only layers: the final-stream queries against all
+keys), Sec. 3.2 (decoding with the expanded KV cache).  The backward is the
+derivative of that forward (the paper does not write it out).
 
 Pinned by ``tests/test_oracle_pins.py``; see the header of ``hdsfa_oracle.c``.
 """
