@@ -22,6 +22,14 @@ def test_visible_pair_model_matches_oracle_mask(n, L):
         assert bench.visible_pairs(s, mode, w) == cnt
 
 
+@pytest.mark.parametrize("n,L", [(1, 9), (2, 7), (4, 5), (3, 6)])
+def test_final_stream_pair_model_matches_oracle_mask(n, L):
+    # the final-stream queries (1-indexed positions t = i*n) against every key position
+    for mode, w in ((WITHIN, 0), (CROSS, 0), (LOCAL, 3), (LOCAL, 100)):
+        count = sum(oracle.visible(i * n, tk, n, mode, w) for i in range(1, L + 1) for tk in range(1, n * L + 1))
+        assert bench.final_pairs(L, n, mode, w) == count, (mode, w)
+
+
 def test_flop_model_headline_workload():
     s = bench.SHAPES[bench.WORKLOAD]
     assert bench.visible_pairs(s, WITHIN) == 33_562_624
