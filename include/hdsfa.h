@@ -100,6 +100,9 @@ hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dta
  * gradient rows into dtables following a plan of the same ids, B, L and V; the
  * workspace must hold that plan, unmodified, when the apply runs (order a plan on
  * another stream before the apply with an event).  plan + apply == hd_expand_embed_bwd.
+ * An apply on a workspace that does not hold such a plan gives meaningless sums but
+ * never reads or writes outside dout, dtables and the workspace: records and token
+ * indexes outside the plan's ranges are skipped.
  */
 hd_status_t hd_expand_embed_bwd_plan(const int32_t* ids, int B, int L, int V, void* workspace,
                                      size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream);

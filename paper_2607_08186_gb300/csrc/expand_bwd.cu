@@ -232,13 +232,18 @@ __global__ void __launch_bounds__(kRowThreads, 3) rows_kernel(const bf16* __rest
                                                           const uint4* __restrict__ light,
                                                           const uint4* __restrict__ heavy,
                                                           const unsigned* __restrict__ counts,
-                                                          float* __restrict__ de, int n, int V, int D) {
+                                                          float* __restrict__ de, long long N, int n, int V,
+                                                          int D) {
   __shared__ float part[kHeavyBlocks][kHeavyItems][9];  // padded against bank conflicts
   const int d8 = D / 8, items = n * d8;
   const long long nD = (long long)n * D;
   const int SL = (items + kLightItems - 1) / kLightItems, SH = (items + kHeavyItems - 1) / kHeavyItems;
   // heavy units first: they take longest, so they start before the light ones
-  const long long hunits = (long long)counts[1] * SH, units = hunits + (long long)counts[0] * SL;
+  // The run lists hold at most N records each; a record or a key outside the plan's
+  // ranges (a workspace the plan did not write) is skipped, so every access stays in
+  // bounds whatever the workspace holds.
+  const long long nl = counts[0] < N ? counts[0] : N, nh = counts[1] < N ? counts[1] : N;
+  const long long hunits = nh * SH, units = hunits + nl * SL;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (long long w = blockIdx.x; w < units; w += gridDim.x) {
     if (w >= hunits) {
@@ -246,6 +251,7 @@ __global__ void __launch_bounds__(kRowThreads, 3) rows_kernel(const bf16* __rest
       const int z = (int)(lw - r * SL);
       const uint4 rec = light[r];
       const uint32_t start = rec.x, m = rec.y, v = rec.w;
+      if (start >= N || m > N - start || v >= (uint32_t)V || rec.z >= N) continue;
       int it[2];
       float* drow[2];
       float4 e0[2], e1[2];
@@ -271,6 +277,7 @@ __global__ void __launch_bounds__(kRowThreads, 3) rows_kernel(const bf16* __rest
           const uint32_t j = j0 + u;
           long long tok = -1;
           if (j < m) tok = j == 0 ? (long long)rec.z : (long long)(uint32_t)keys[start + j];
+          if (tok >= N) tok = -1;
 #pragma unroll
           for (int q = 0; q < 2; ++q) {
             x[u][q] = make_uint4(0, 0, 0, 0);
@@ -293,6 +300,7 @@ __global__ void __launch_bounds__(kRowThreads, 3) rows_kernel(const bf16* __rest
       const int z = (int)(w - r * SH);
       const uint4 rec = heavy[r];
       const uint32_t start = rec.x, m = rec.y, v = rec.w;
+      if (start >= N || m > N - start || v >= (uint32_t)V) continue;  // uniform over the block
       const int itm = z * kHeavyItems + lane;
       const bool live = itm < items;
       // token block of this warp: [m*warp/8, m*(warp+1)/8)
@@ -306,7 +314,7 @@ __global__ void __launch_bounds__(kRowThreads, 3) rows_kernel(const bf16* __rest
           x[u] = make_uint4(0, 0, 0, 0);
           if (j0 + u < je && live) {
             const long long tok = (long long)(uint32_t)keys[start + j0 + u];
-            x[u] = *reinterpret_cast<const uint4*>(dx + tok * nD + (long long)itm * 8);
+            if (tok < N) x[u] = *reinterpret_cast<const uint4*>(dx + tok * nD + (long long)itm * 8);
           }
         }
 #pragma unroll
@@ -431,7 +439,8 @@ cudaError_t launch_expand_bwd_apply(const void* dx, float* de, int B, int L, int
                                     cudaStream_t st) {
   using namespace ebwd;
   const ExpandBwdWs w = split_ws(const_cast<void*>(ws), (long long)B * L);
-  rows_kernel<<<152 * 3, kRowThreads, 0, st>>>((const bf16*)dx, w.keys, w.light, w.heavy, w.counts, de, n, V, D);
+  rows_kernel<<<152 * 3, kRowThreads, 0, st>>>((const bf16*)dx, w.keys, w.light, w.heavy, w.counts, de,
+                                                 (long long)B * L, n, V, D);
   return cudaGetLastError();
 }
 

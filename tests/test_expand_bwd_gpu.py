@@ -130,6 +130,27 @@ def test_plan_once_apply_twice_on_another_stream():
     assert torch.equal(one.view(torch.int32), dE2.cpu().view(torch.int32))
 
 
+def test_apply_skips_what_the_plan_does_not_cover():
+    # a plan for V = 300 applied to tables of V = 150 rows: ids >= 150 contribute nothing
+    # and the rest sum as usual; a workspace of random bytes (no plan at all) gives
+    # meaningless sums but every access stays inside the buffers
+    B, L, n, V, D = 2, 700, 4, 300, 128
+    ids = inputs.token_ids(B, L, V, seed=18, zipf=1.0)
+    dX = inputs.normal_bf16((B, n * L, D), seed=19)
+    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device="cuda")
+    binding.hd_expand_embed_bwd_plan(ids.cuda(), V, ws)
+    dE = torch.zeros(n, 150, D, dtype=torch.float32, device="cuda")
+    binding.hd_expand_embed_bwd_apply(dX.cuda(), dE, ws, L)
+    torch.cuda.synchronize()
+    _check_sum(dE.cpu(), dX, ids, n, 150)
+    g = torch.Generator().manual_seed(20)
+    ws.copy_(torch.randint(0, 256, (ws.numel(),), dtype=torch.uint8, generator=g))
+    dE.zero_()
+    binding.hd_expand_embed_bwd_apply(dX.cuda(), dE, ws, L)
+    torch.cuda.synchronize()
+    assert bool(torch.isfinite(dE).all())
+
+
 def test_deterministic_bits():
     B, L, n, V, D = 2, 3000, 4, 50, 512
     dX = inputs.normal_bf16((B, n * L, D), seed=12)
