@@ -52,6 +52,14 @@ struct DecodeArgs {
   float scale_log2;
 };
 
+// Programmatic dependent launch: both kernels are launched so that they may start
+// while the kernel before them in the stream is finishing; each waits for that
+// kernel's results before its first read of them, and the decode kernel lets the
+// combine kernel launch at once, so the combine's launch and start overlap the
+// decode's tail.  Without the launch attribute both are no-ops.
+HD_DEVINLINE void grid_dep_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+HD_DEVINLINE void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
 // Visible position range [lo, hi) of a sequence of T tokens (the new token's rows
 // see nothing outside it; per-row conditions are applied per element).
 HD_DEVINLINE void seq_range(const DecodeArgs& a, int T, int& lo, int& hi) {
@@ -71,6 +79,8 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
   const size_t pidx = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit + c;
   float* po = a.part_o + pidx * RG * DH;
   float2* pml = a.part_ml + pidx * RG;
+  grid_dep_wait();
+  grid_dep_launch();
   const int T = a.lens[b];
   int k0 = 0, k1 = 0;
   if (T >= 1 && T <= a.maxT) {
@@ -295,6 +305,7 @@ __global__ void __launch_bounds__(256) combine_kernel(DecodeArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rows = min(RG, a.M - rg * RG);
   const size_t pidx0 = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit;
+  grid_dep_wait();  // every partial of the decode kernel is written
   const int T = a.lens[b];
   const bool valid = T >= 1 && T <= a.maxT;
   if (!valid && blockIdx.x == 0 && c8 == 0 && threadIdx.x == 0) set_status(a.status, HD_DEVBIT_INDEX);
@@ -414,11 +425,22 @@ static cudaError_t launch_decode_t(const dec::DecodeArgs& a, cudaStream_t st) {
   const size_t smem = (size_t)(MT * 16 + 2 * STAGES * KT) * DH * sizeof(bf16);
   cudaError_t e = cudaFuncSetAttribute(decode_kernel<DH, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  decode_kernel<DH, MT><<<dim3(a.nsplit, a.Hkv * a.ngroups, a.B), NT, smem, st>>>(a);
-  e = cudaGetLastError();
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.nsplit, a.Hkv * a.ngroups, a.B);
+  cfg.blockDim = dim3(NT);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = pdl;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, decode_kernel<DH, MT>, a);
   if (e != cudaSuccess) return e;
-  combine_kernel<DH><<<dim3(a.Hkv * a.ngroups, a.B, DH / 8), 256, 0, st>>>(a);
-  return cudaGetLastError();
+  cfg.gridDim = dim3(a.Hkv * a.ngroups, a.B, DH / 8);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = 0;
+  return cudaLaunchKernelEx(&cfg, combine_kernel<DH>, a);
 }
 
 cudaError_t launch_sfa_decode(const void* q, const void* kc, const void* vc, const int32_t* lens, void* o,
