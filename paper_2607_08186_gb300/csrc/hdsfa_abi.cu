@@ -29,6 +29,8 @@ cudaError_t launch_kv_append(const void* kn, const void* vn, void* kc, void* vc,
                              int Lcap, int n, int Hkv, int Dh, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
                               const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
+cudaError_t launch_sfa_fwd_tc256(const void* q, const void* k, const void* v, void* o, float* lse,
+                                 const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
                                const SfaGeom& g, int Dh, float scale, cudaStream_t st);
 cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
@@ -234,10 +236,9 @@ hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float*
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  // head dim 256 (no room for its O and S accumulators beside a second query tile in
-  // TMEM) runs on the mma.sync kernel
-  if (use_mma_kernels() || Dh == 256)
-    return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  if (use_mma_kernels()) return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  // head dim 256: one query tile per CTA (its O takes half of TMEM)
+  if (Dh == 256) return cuda_status(hdsfa::launch_sfa_fwd_tc256(q, k, v, o, lse, g, scale, dev_status, stream));
   return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
 }
 
@@ -395,8 +396,8 @@ hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, 
   hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  if (use_mma_kernels() || Dh == 256)  // head dim 256: the mma.sync kernel, as in sfa_fwd
-    return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  if (use_mma_kernels()) return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
+  if (Dh == 256) return cuda_status(hdsfa::launch_sfa_fwd_tc256(q, k, v, o, lse, g, scale, dev_status, stream));
   return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
 }
 

@@ -66,10 +66,18 @@ def test_wide_gqa_groups(mode, window):
 
 @pytest.mark.parametrize("mode,window", [(WITHIN, 0), (CROSS, 0), (LOCAL, 40)])
 def test_head_dim_256(mode, window):
-    # head dim 256 (the paper's 80B configuration, 24 query over 2 K/V heads, Table 6) on
-    # the mma.sync kernels: the backward in two launches over halves of the head dim
+    # head dim 256 (the paper's 80B configuration, 24 query over 2 K/V heads, Table 6):
+    # the forward on its own tcgen05 kernel, the backward on the mma.sync kernel in two
+    # launches over halves of the head dim
     _full_case(AttnShape(1, 70, 4, 24, 2, 256), mode, seed=31, window=window)
     _full_case(AttnShape(2, 33, 2, 4, 4, 256), mode, seed=32, window=window)
+
+
+@pytest.mark.parametrize("mode,window", [(WITHIN, 0), (CROSS, 0), (LOCAL, 333)])
+def test_head_dim_256_many_key_tiles(mode, window):
+    # 1200 positions: up to 10 key tiles per query tile, so the head-dim-256 forward's
+    # five-slot K/V ring wraps several times; ragged last tiles (1200 = 9*128 + 48)
+    _full_case(AttnShape(1, 300, 4, 4, 2, 256), mode, seed=33, window=window)
 
 
 @pytest.mark.parametrize("window", [1, 50, 200])
@@ -178,6 +186,12 @@ def test_qwen3_8b_class_layer(mode):
 def test_large_moe_class_layer(mode):
     # B=1, L=8192, n=4 (32768 positions), Hq=64, Hkv=8, Dh=128
     _sampled_parity(inputs.SHAPES["moe_large_n4"], mode, seed=21, n_rows=96, n_kv=24)
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_80b_class_layer(mode):
+    # B=1, L=4096, n=4 (16384 positions), Hq=24, Hkv=2, Dh=256 (Table 6's 80B heads)
+    _sampled_parity(AttnShape(1, 4096, 4, 24, 2, 256), mode, seed=51, n_rows=64, n_kv=16)
 
 
 @pytest.mark.parametrize("n", [1, 2, 8])
