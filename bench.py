@@ -641,6 +641,9 @@ def main():
     ap.add_argument("--layer-only", choices=["within", "cross", "local"], default=None,
                     help="time only one attention layer (fwd + bwd, no gather / e2e / extras); "
                          "the small case used for kernel profiles")
+    ap.add_argument("--head-dim", type=int, choices=[128, 256], default=128,
+                    help="with --layer-only: 128 = the Qwen3-8B-class layer, 256 = the 80B-class "
+                         "layer (B=1, L=4096, n=4, Hq=24, Hkv=2)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     ws, rank, local = dist_setup()
@@ -680,11 +683,13 @@ def main():
     if args.layer_only:
         mode = {"within": WITHIN, "cross": CROSS, "local": LOCAL}[args.layer_only]
         w = 4096 if mode == LOCAL else 0
-        r = measure_layer(s, mode, dev, iters=args.steps, warmup=args.warmup, window=w)
-        fl = attn_flops(s, mode, FWD_FLOP + BWD_FLOP, w)
+        ls, name = (s, WORKLOAD) if args.head_dim == 128 else (AttnShape(1, 4096, 4, 24, 2, 256), "80b_dh256_n4")
+        r = measure_layer(ls, mode, dev, iters=args.steps, warmup=args.warmup, window=w)
+        fl = attn_flops(ls, mode, FWD_FLOP + BWD_FLOP, w)
         if rank == 0:
-            print(json.dumps({"layer": f"{WORKLOAD}_{args.layer_only}", "ms": r["step_s"] * 1e3,
+            print(json.dumps({"layer": f"{name}_{args.layer_only}", "ms": r["step_s"] * 1e3,
                               "tflops": fl / r["step_s"] / 1e12, "fwd_ms": r["fwd_s"] * 1e3,
+                              "fwd_tflops": attn_flops(ls, mode, FWD_FLOP, w) / r["fwd_s"] / 1e12,
                               "bwd_main_ms": r["bwd_main_s"] * 1e3}), flush=True)
         return
     hp = HotPath(s, WITHIN, dev, with_gather=True, seed=1)
