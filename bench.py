@@ -484,43 +484,49 @@ def measure_final_layer(dev, bf16_peak: float, iters: int = 5):
 
 
 def measure_decode(dev, hbm_peak: float, quick: bool = False):
-    """Decoding step (Sec. 3.2) with Qwen3-8B-class heads (Hq=32, Hkv=8, Dh=128), n=4:
-    the new token's 4 positions against a context of T tokens (4T cached positions) for
-    batch B, WITHIN and CROSS layers.  Algorithmic bytes: the visible cached K and V rows
-    (B*T*n*Hkv*Dh*2 bytes each) plus q and o; rotating cache sets keep every call out of L2."""
+    """Decoding step (Sec. 3.2), n=4: the new token's 4 positions against a context of T
+    tokens (4T cached positions) for batch B, WITHIN and CROSS layers, with Qwen3-8B-class
+    heads (Hq=32, Hkv=8, Dh=128) and, unless quick, 80B-class heads (Hq=24, Hkv=2, Dh=256,
+    Table 6).  Algorithmic bytes: the visible cached K and V rows (B*T*n*Hkv*Dh*2 bytes
+    each) plus q and o; rotating cache sets keep every call out of L2."""
     from paper_2607_08186_gb300 import binding
-    n, Hq, Hkv, Dh = 4, 32, 8, 128
-    grid = [(1, 8192), (4, 8192), (16, 8192), (1, 32768), (16, 32768)]
+    n = 4
+    heads = {"qwen3_8b": (32, 8, 128, [(1, 8192), (4, 8192), (16, 8192), (1, 32768), (16, 32768)]),
+             "80b": (24, 2, 256, [(1, 8192), (16, 8192), (1, 32768), (16, 32768)])}
     if quick:
-        grid = [(1, 8192), (16, 8192)]
-    out = []
+        heads = {"qwen3_8b": (32, 8, 128, [(1, 8192), (16, 8192)])}
+    res = {}
     g = torch.Generator(device=dev)
     g.manual_seed(41)
-    for B, T in grid:
-        cache_bytes = 2 * B * T * n * Hkv * Dh * 2
-        S = max(1, min(3, -(-400_000_000 // cache_bytes)))
-        sets = []
-        for _ in range(S):
-            kc = torch.randn(B, T * n, Hkv, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
-            vc = torch.randn(B, T * n, Hkv, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
-            q = torch.randn(B, n, Hq, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
-            sets.append((q, kc, vc))
-        lens = torch.full((B,), T, dtype=torch.int32, device=dev)
-        o = torch.empty(B, n, Hq, Dh, dtype=torch.bfloat16, device=dev)
-        lse = torch.empty(B, Hq, n, dtype=torch.float32, device=dev)
-        row = {"B": B, "context_tokens": T, "cached_positions": T * n}
-        for mode in (WITHIN, CROSS):
-            ws = torch.empty(binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
-                             device=dev)
-            t = time_op(lambda k: binding.sfa_decode(sets[k][0], sets[k][1], sets[k][2], lens, o, n, mode, ws,
-                                                     max_tokens=T, lse=lse), S)
-            nbytes = cache_bytes + 2 * B * n * Hq * Dh * 2
-            row[MODE_NAME[mode]] = {"us": t * 1e6, "gbs": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / hbm_peak}
-        out.append(row)
-        del sets, o, lse
-        torch.cuda.empty_cache()
-    return {"workload": "decode step, Hq=32 Hkv=8 Dh=128 n=4, all sequences at the context length; "
-                        "bytes = cached K+V rows read + q + o", "rows": out}
+    for name, (Hq, Hkv, Dh, grid) in heads.items():
+        out = []
+        for B, T in grid:
+            cache_bytes = 2 * B * T * n * Hkv * Dh * 2
+            S = max(1, min(3, -(-400_000_000 // cache_bytes)))
+            sets = []
+            for _ in range(S):
+                kc = torch.randn(B, T * n, Hkv, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+                vc = torch.randn(B, T * n, Hkv, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+                q = torch.randn(B, n, Hq, Dh, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+                sets.append((q, kc, vc))
+            lens = torch.full((B,), T, dtype=torch.int32, device=dev)
+            o = torch.empty(B, n, Hq, Dh, dtype=torch.bfloat16, device=dev)
+            lse = torch.empty(B, Hq, n, dtype=torch.float32, device=dev)
+            row = {"B": B, "context_tokens": T, "cached_positions": T * n}
+            for mode in (WITHIN, CROSS):
+                ws = torch.empty(binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
+                                 device=dev)
+                t = time_op(lambda k: binding.sfa_decode(sets[k][0], sets[k][1], sets[k][2], lens, o, n, mode, ws,
+                                                         max_tokens=T, lse=lse), S)
+                nbytes = cache_bytes + 2 * B * n * Hq * Dh * 2
+                row[MODE_NAME[mode]] = {"us": t * 1e6, "gbs": nbytes / t / 1e9,
+                                        "frac_hbm": nbytes / t / 1e9 / hbm_peak}
+            out.append(row)
+            del sets, o, lse
+            torch.cuda.empty_cache()
+        res[name] = {"heads": f"Hq={Hq} Hkv={Hkv} Dh={Dh}", "rows": out}
+    return {"workload": "decode step, n=4, all sequences at the context length; "
+                        "bytes = cached K+V rows read + q + o", **res}
 
 
 # ---------------------------------------------------------------- ncu traffic record

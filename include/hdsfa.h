@@ -239,8 +239,8 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
  *   workspace: device memory of >= sfa_decode_workspace_bytes(B, max_tokens, n, Hq,
  *              Hkv, Dh, mode, window) bytes, 16-byte aligned (partial results).
  * A sequence with lens outside [1, max_tokens] gets zero rows, LSE = -inf and
- * HD_DEVBIT_INDEX.  Dh in {64, 128}; Lcap*n <= 2^30.  HBM-bound (reads the visible
- * cached rows once per step).
+ * HD_DEVBIT_INDEX.  Dh in {64, 128, 256}; Lcap*n <= 2^30.  HBM-bound (reads the
+ * visible cached rows once per step).
  */
 size_t sfa_decode_workspace_bytes(int B, int max_tokens, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode,
                                   int window); /* 0 for invalid sizes */

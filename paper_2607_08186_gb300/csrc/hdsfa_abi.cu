@@ -348,7 +348,7 @@ static hd_status_t decode_sizes(int B, int maxT, int Lcap, int n, int Hq, int Hk
   if (Hq % Hkv != 0 || maxT > Lcap) return HD_ERR_INVALID_ARG;
   if (mode != SFA_WITHIN && mode != SFA_CROSS && mode != SFA_LOCAL) return HD_ERR_INVALID_ARG;
   if (mode == SFA_LOCAL && window <= 0) return HD_ERR_INVALID_ARG;
-  if (Dh != 64 && Dh != 128) return HD_ERR_UNSUPPORTED;
+  if (Dh != 64 && Dh != 128 && Dh != 256) return HD_ERR_UNSUPPORTED;
   if ((long long)Lcap * n > (1LL << 30) || (long long)n * Hq > (1LL << 20)) return HD_ERR_UNSUPPORTED;
   return HD_OK;
 }

@@ -18,6 +18,9 @@
 //                   ring of 64-position K/V tiles; warp w takes keys [16w, 16w+16) of
 //                   each tile with its own online softmax; the 4 warps merge in shared
 //                   memory and write an unnormalised partial (O, running max, sum).
+//                   At head dim 256 the tiles are 32 positions and the warps pair up:
+//                   both warps of a pair compute the same scores and softmax for their
+//                   16 keys, each accumulates O for one half of the head dim.
 //   combine_kernel: merges a row's partials, writes O (bf16) and the natural-log LSE.
 // Masking is per element (the new token's own positions, the stream condition of an
 // intra-stream layer, the window); rows past the group's query count and positions
@@ -33,8 +36,14 @@ typedef __nv_bfloat16 bf16;
 
 namespace dec {
 constexpr int NT = 128;      // 4 warps
-constexpr int KT = 64;       // cached positions per pipeline stage
 constexpr int STAGES = 3;
+// Head-dim split of the warps: at head dim 256 the four warps form two key groups x two
+// halves of the head dim (a warp's O accumulator would not fit its registers whole);
+// otherwise four key groups.  A stage holds 16 cached positions per key group.
+template <int DH>
+constexpr int dsplit() { return DH == 256 ? 2 : 1; }
+template <int DH>
+constexpr int ktile() { return 64 / dsplit<DH>(); }  // cached positions per pipeline stage
 constexpr int RG = 32;       // query rows per CTA at most (two m16 tiles)
 constexpr int kMaxSplit = 128;
 
@@ -69,6 +78,7 @@ HD_DEVINLINE void seq_range(const DecodeArgs& a, int T, int& lo, int& hi) {
 
 template <int DH, int MT>
 __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
+  constexpr int DS = dsplit<DH>(), KT = ktile<DH>(), KW = 4 / DS, DC = DH / DS;  // DC: O columns per warp
   extern __shared__ __align__(128) uint8_t smem_raw[];
   bf16* sQ = reinterpret_cast<bf16*>(smem_raw);  // [MT*16][DH]
   bf16* sK = sQ + MT * 16 * DH;                   // [STAGES][KT][DH]
@@ -76,6 +86,7 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
   constexpr int CPR = DH / 8;
   const int c = blockIdx.x, g = blockIdx.y / a.ngroups, rg = blockIdx.y % a.ngroups, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g4 = lane >> 2, t4 = lane & 3;
+  const int kw = warp / DS, dw = warp % DS;  // key group and head-dim part of this warp
   const size_t pidx = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit + c;
   float* po = a.part_o + pidx * RG * DH;
   float2* pml = a.part_ml + pidx * RG;
@@ -138,13 +149,13 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
   for (int j = 0; j < 2; ++j)
 #pragma unroll
     for (int e = 0; e < 2; ++e) kst0[j][e] = (j * 8 + 2 * t4 + e) % a.n;
-  float mx[MT][2], ls[MT][2], oacc[MT][DH / 8][4];
+  float mx[MT][2], ls[MT][2], oacc[MT][DC / 8][4];
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
     mx[mt][0] = mx[mt][1] = -INFINITY;
     ls[mt][0] = ls[mt][1] = 0.f;
 #pragma unroll
-    for (int i = 0; i < DH / 8; ++i) oacc[mt][i][0] = oacc[mt][i][1] = oacc[mt][i][2] = oacc[mt][i][3] = 0.f;
+    for (int i = 0; i < DC / 8; ++i) oacc[mt][i][0] = oacc[mt][i][1] = oacc[mt][i][2] = oacc[mt][i][3] = 0.f;
   }
 
   for (int it = 0; it < nsub; ++it) {
@@ -163,7 +174,7 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
 #pragma unroll
     for (int kk = 0; kk < DH / 16; ++kk) {
       uint32_t b0, b1, b2, b3;
-      ldsm_x4(smem_u32(cK + swz<DH>(warp * 16 + (lane & 7) + (lane >> 4) * 8, kk * 16 + ((lane >> 3) & 1) * 8)),
+      ldsm_x4(smem_u32(cK + swz<DH>(kw * 16 + (lane & 7) + (lane >> 4) * 8, kk * 16 + ((lane >> 3) & 1) * 8)),
               b0, b1, b2, b3);
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
@@ -175,7 +186,7 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
       }
     }
     // mask + online softmax (log2 domain)
-    const int kb = k0 + it * KT + warp * 16;
+    const int kb = k0 + it * KT + kw * 16;
     int kp[2][2], kst[2][2];
 #pragma unroll
     for (int j = 0; j < 2; ++j)
@@ -219,7 +230,7 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
           ls[mt][e4 >> 1] += p;
         }
 #pragma unroll
-      for (int i = 0; i < DH / 8; ++i) {
+      for (int i = 0; i < DC / 8; ++i) {
         oacc[mt][i][0] *= corr[0];
         oacc[mt][i][1] *= corr[0];
         oacc[mt][i][2] *= corr[1];
@@ -236,9 +247,10 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
       pa[mt][3] = pack_bf16(sacc[mt][1][2], sacc[mt][1][3]);
     }
 #pragma unroll
-    for (int dp = 0; dp < DH / 16; ++dp) {
+    for (int dp = 0; dp < DC / 16; ++dp) {
       uint32_t b0, b1, b2, b3;
-      ldsm_x4_t(smem_u32(cV + swz<DH>(warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8, dp * 16 + (lane >> 4) * 8)),
+      ldsm_x4_t(smem_u32(cV + swz<DH>(kw * 16 + (lane & 7) + ((lane >> 3) & 1) * 8,
+                                      dw * DC + dp * 16 + (lane >> 4) * 8)),
                 b0, b1, b2, b3);
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
@@ -251,9 +263,12 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
   // merge the 4 warps' partials in shared memory (the K/V ring is free now)
   cp_async_wait<0>();
   __syncthreads();
-  float* sO = reinterpret_cast<float*>(sK);  // [4][MT*16][DH]
-  float* sM = sO + 4 * MT * 16 * DH;         // [4][MT*16]
-  float* sL = sM + 4 * MT * 16;              // [4][MT*16]
+  // [KW][MT*16][DH]: key group kw's O, its head-dim parts side by side; then the key
+  // groups' running max and sum (the DS warps of a key group hold the same ones)
+  static_assert((KW * MT * 16 * DH + 2 * KW * MT * 16) * 4 <= 2 * STAGES * KT * DH * 2, "merge fits the ring");
+  float* sO = reinterpret_cast<float*>(sK);
+  float* sM = sO + KW * MT * 16 * DH;  // [KW][MT*16]
+  float* sL = sM + KW * MT * 16;       // [KW][MT*16]
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
 #pragma unroll
@@ -261,17 +276,17 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
       ls[mt][hf] += __shfl_xor_sync(0xffffffffu, ls[mt][hf], 1);
       ls[mt][hf] += __shfl_xor_sync(0xffffffffu, ls[mt][hf], 2);
       const int row = mt * 16 + g4 + 8 * hf;
-      if (t4 == 0) {
-        sM[warp * MT * 16 + row] = mx[mt][hf];
-        sL[warp * MT * 16 + row] = ls[mt][hf];
+      if (t4 == 0 && dw == 0) {
+        sM[kw * MT * 16 + row] = mx[mt][hf];
+        sL[kw * MT * 16 + row] = ls[mt][hf];
       }
     }
 #pragma unroll
-    for (int i = 0; i < DH / 8; ++i)
+    for (int i = 0; i < DC / 8; ++i)
 #pragma unroll
       for (int e4 = 0; e4 < 4; ++e4) {
-        const int row = mt * 16 + g4 + 8 * (e4 >> 1), col = i * 8 + 2 * t4 + (e4 & 1);
-        sO[(warp * MT * 16 + row) * DH + col] = oacc[mt][i][e4];
+        const int row = mt * 16 + g4 + 8 * (e4 >> 1), col = dw * DC + i * 8 + 2 * t4 + (e4 & 1);
+        sO[(kw * MT * 16 + row) * DH + col] = oacc[mt][i][e4];
       }
   }
   __syncthreads();
@@ -279,11 +294,11 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
     const int row = idx / DH, col = idx % DH;
     float m = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) m = fmaxf(m, sM[w * MT * 16 + row]);
+    for (int w = 0; w < KW; ++w) m = fmaxf(m, sM[w * MT * 16 + row]);
     float o = 0.f, l = 0.f;
     if (m != -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
+      for (int w = 0; w < KW; ++w) {
         const float mw = sM[w * MT * 16 + row];
         const float f = mw == -INFINITY ? 0.f : exp2f(mw - m);
         o += f * sO[(w * MT * 16 + row) * DH + col];
@@ -393,9 +408,11 @@ DecodePlan decode_plan(int B, int maxT, int n, int Hq, int Hkv, int Dh, int mode
   p.ngroups = (p.M + RG - 1) / RG;
   const long long range = mode == SFA_LOCAL ? std::min<long long>((long long)maxT * n, (long long)window + n - 1)
                                             : (long long)maxT * n;
+  const int KT = Dh == 256 ? ktile<256>() : ktile<128>();
   const long long tiles = (range + KT - 1) / KT;
   const long long ctas = (long long)B * Hkv * p.ngroups;
-  // resident decode CTAs: two per SM at head dim 128 (104 KB of shared memory), four at 64
+  // resident decode CTAs: two per SM at head dim 128 (104 KB of shared memory) and 256
+  // (112 KB), four at 64
   const long long resident = 152LL * (Dh == 64 ? 4 : 2);
   // split count: least (waves x (tiles per CTA + a fixed cost of about two tiles))
   long long best = 1, best_cost = -1;
@@ -422,7 +439,7 @@ size_t decode_ws_bytes(const DecodePlan& p) { return ((p.part_o_bytes + 255) & ~
 template <int DH, int MT>
 static cudaError_t launch_decode_t(const dec::DecodeArgs& a, cudaStream_t st) {
   using namespace dec;
-  const size_t smem = (size_t)(MT * 16 + 2 * STAGES * KT) * DH * sizeof(bf16);
+  const size_t smem = (size_t)(MT * 16 + 2 * STAGES * ktile<DH>()) * DH * sizeof(bf16);
   cudaError_t e = cudaFuncSetAttribute(decode_kernel<DH, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchAttribute pdl[1];
@@ -473,6 +490,7 @@ cudaError_t launch_sfa_decode(const void* q, const void* kc, const void* vc, con
   a.scale_log2 = scale * 1.4426950408889634f;
   const bool two = p.M > 16;  // a row group of more than 16 rows takes two m16 tiles
   if (Dh == 64) return two ? launch_decode_t<64, 2>(a, st) : launch_decode_t<64, 1>(a, st);
+  if (Dh == 256) return two ? launch_decode_t<256, 2>(a, st) : launch_decode_t<256, 1>(a, st);
   return two ? launch_decode_t<128, 2>(a, st) : launch_decode_t<128, 1>(a, st);
 }
 

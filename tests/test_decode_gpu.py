@@ -71,6 +71,16 @@ def test_shapes_ragged(mode, w, n, Hq, Hkv):
     _check(q, kc, vc, torch.tensor([Lcap, 1, 129], dtype=torch.int32), n, mode, w)
 
 
+@pytest.mark.parametrize("mode,w", [(WITHIN, 0), (CROSS, 0), (LOCAL, 1), (LOCAL, 100)])
+@pytest.mark.parametrize("n,Hq,Hkv", [(4, 24, 2), (4, 4, 1), (3, 6, 2)])
+def test_head_dim_256_ragged(mode, w, n, Hq, Hkv):
+    # head dim 256 (Table 6's 80B heads: 24 query over 2 K/V heads, 48 query rows per K/V
+    # head in two row groups), one m16 tile, and 9 rows; lengths 1, 129 and the capacity
+    Lcap = 300
+    q, kc, vc = _case(3, Lcap, n, Hq, Hkv, 256, 40 + n + Hq)
+    _check(q, kc, vc, torch.tensor([Lcap, 1, 129], dtype=torch.int32), n, mode, w)
+
+
 def test_max_tokens_below_capacity():
     q, kc, vc = _case(2, 500, 4, 8, 2, 128, 5)
     _check(q, kc, vc, torch.tensor([200, 77], dtype=torch.int32), 4, CROSS, max_tokens=200)
@@ -105,6 +115,14 @@ def test_full_size(mode):
     _check(q, kc, vc, torch.tensor([8192, 5000], dtype=torch.int32), 4, mode)
 
 
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_full_size_head_dim_256(mode):
+    # 80B-class heads (Hq=24, Hkv=2, Dh=256), n = 4, an 8192-token context, B = 2 with one
+    # shorter sequence; every output row checked against the oracle
+    q, kc, vc = _case(2, 8192, 4, 24, 2, 256, 18)
+    _check(q, kc, vc, torch.tensor([8192, 3001], dtype=torch.int32), 4, mode)
+
+
 def test_kv_append_bit_exact_and_flag():
     B, n, Lcap, Hkv, Dh = 4, 4, 33, 8, 128
     kc = inputs.normal_bf16((B, Lcap * n, Hkv, Dh), 9)
@@ -124,10 +142,11 @@ def test_kv_append_bit_exact_and_flag():
     assert torch.equal(vd.cpu().view(torch.int16), v_ref.view(torch.int16))
 
 
-def test_append_then_decode_equals_forward_rows():
+@pytest.mark.parametrize("Hq,Hkv,Dh", [(8, 2, 128), (24, 2, 256)])
+def test_append_then_decode_equals_forward_rows(Hq, Hkv, Dh):
     # a prefilled cache (the forward's K/V) plus one appended token decodes to the
     # forward's rows of that token, for every mask
-    B, L, n, Hq, Hkv, Dh = 1, 50, 4, 8, 2, 128
+    B, L, n = 1, 50, 4
     q, k, v = inputs.attn_inputs(inputs.AttnShape(B, L, n, Hq, Hkv, Dh), seed=13, with_grad=False)
     kd = torch.zeros(B, L * n, Hkv, Dh, dtype=torch.bfloat16, device="cuda")
     vd = torch.zeros_like(kd)
