@@ -40,20 +40,21 @@ if ROOT not in sys.path:
 
 import torch  # noqa: E402
 
-from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, SHAPES, WITHIN, attn_inputs  # noqa: E402
+from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, SHAPES, WITHIN, WITHIN_NAIVE, attn_inputs  # noqa: E402
 
 METRIC = "SFA fwd+bwd TFLOP/s (visible pairs) at n=4, % of bf16 peak; scaling vs n"
 WORKLOAD = "qwen3_8b_n4"
 GATHER_V, GATHER_D = 151936, 4096
 FWD_FLOP, BWD_FLOP = 4, 10  # per visible pair, per query head, times Dh
-MODE_NAME = {WITHIN: "WITHIN", CROSS: "CROSS", LOCAL: "LOCAL"}
+MODE_NAME = {WITHIN: "WITHIN", CROSS: "CROSS", LOCAL: "LOCAL", WITHIN_NAIVE: "WITHIN_naive"}
 
 
 # ---------------------------------------------------------------- FLOP model
 def visible_pairs(s: AttnShape, mode: int, window: int = 0) -> int:
     """Visible (query, key) pairs per (batch, head): WITHIN n*L(L+1)/2 (Eq. 4),
-    CROSS nL(nL+1)/2 (Fig. 2a), LOCAL sum_p min(p+1, w) (Fig. 2b)."""
-    if mode == WITHIN:
+    CROSS nL(nL+1)/2 (Fig. 2a), LOCAL sum_p min(p+1, w) (Fig. 2b).  The naive WITHIN
+    schedule computes the WITHIN result: its pairs are WITHIN's."""
+    if mode in (WITHIN, WITHIN_NAIVE):
         return s.n * s.L * (s.L + 1) // 2
     if mode == CROSS:
         return s.nL * (s.nL + 1) // 2
@@ -532,7 +533,7 @@ def measure_decode(dev, hbm_peak: float, quick: bool = False):
 # ---------------------------------------------------------------- ncu traffic record
 # ABI phase -> (kernel symbol, source file) of the implementation the library runs.
 KERNEL_OF = {
-    "sfa_fwd": ("hdsfa::tcfwd::fwd_kernel<128>", "sfa_fwd_tc.cu"),
+    "sfa_fwd": ("hdsfa::tcfwd::fwd_kernel<128, false>", "sfa_fwd_tc.cu"),
     "sfa_bwd_main": ("hdsfa::tcbwd::bwd_kernel<false>", "sfa_bwd_tc.cu"),
 }
 if os.environ.get("HDSFA_KERNELS") == "mma":
@@ -755,6 +756,9 @@ def main():
                    "l2": "inputs larger than L2 (Q 134 MB, dO 134 MB, K+V 67 MB, gather tables 5 GB)",
                    "parallelism": f"replicas x{ws}"},
         "pct_of_peak": 100.0 * value / 1e12 / pk["bf16"],
+        # the same step counted without the backward's QK^T recompute (bwd 8*Dh per pair)
+        "strict_flop_model": {"per_pair": "fwd 4*Dh + bwd 8*Dh", "value": value / 1e12 * 12 / 14,
+                              "unit": "TFLOP/s"},
         "roofline": {"kernel": f"{dom} ({KERNEL_OF[dom][0]})", "bound": "tensor", "achieved": achieved, "peak": pk["bf16"],
                      "unit": "TFLOP/s", "frac": achieved / pk["bf16"],
                      "frac_of_sustained": achieved / pk["bf16_sustained"],
@@ -778,10 +782,13 @@ def main():
         for n in (1, 2, 4, 8):
             sn = AttnShape(1, 4096, n, 32, 8, 128)
             row = {"n": n}
-            for mode in (WITHIN, CROSS):
+            # WITHIN_naive: WITHIN's mask per pair over the full causal tile schedule (no
+            # stream-tile skipping), FLOPs counted over WITHIN's visible pairs
+            for mode in (WITHIN, CROSS, WITHIN_NAIVE):
                 r = measure_layer(sn, mode, dev, iters=3, warmup=1)
                 fl = attn_flops(sn, mode, FWD_FLOP + BWD_FLOP)
                 row[MODE_NAME[mode]] = {"ms": r["step_s"] * 1e3, "tflops": fl / r["step_s"] / 1e12}
+            row["skipping_speedup"] = row["WITHIN_naive"]["ms"] / row["WITHIN"]["ms"]
             sweep.append(row)
         base = sweep[0]["WITHIN"]["ms"]
         for row in sweep:

@@ -54,7 +54,12 @@ typedef enum {
 typedef enum {
   SFA_WITHIN = 0, /* intra-stream: p' <= p and p' = p (mod n)                 (Eq. 4, Fig. 2c) */
   SFA_CROSS = 1,  /* full cross-stream: standard causal mask over nL, p' <= p (Fig. 2a)        */
-  SFA_LOCAL = 2   /* local cross-stream: causal window, p - window < p' <= p  (Fig. 2b)        */
+  SFA_LOCAL = 2,  /* local cross-stream: causal window, p - window < p' <= p  (Fig. 2b)        */
+  SFA_WITHIN_NAIVE = 3 /* measurement mode: the SFA_WITHIN result (same mask, same outputs)
+                          computed over the full causal tile schedule of nL positions, with
+                          the stream condition applied per pair instead of skipping the
+                          other streams' tiles: n times the work, what the skipping saves.
+                          sfa_fwd / sfa_bwd (and their parts) at Dh = 128 only.          */
 } sfa_mode_t;
 
 /*

@@ -31,6 +31,9 @@ struct SfaGeom {
   int qstep, qoff;         // query row r sits at key row r*qstep + qoff (1, 0)
   int q_nL, q_ns, q_rs;    // rows per batch, problems, row step of the query tensors (nL, ns, rs)
   int kv_s0;               // stream of the first key problem (0)
+  int smod;                // > 1: a pair is visible only if its key and query rows are
+                           // congruent mod smod (the intra-stream mask of Eq. 4 over the
+                           // CROSS schedule, SFA_WITHIN_NAIVE); 0 otherwise
 };
 
 // Geometry of the query-side tensors (Q, O, dO, dQ, LSE, row terms) of a problem.

@@ -53,13 +53,18 @@ namespace {
 bool aligned16(const void* p) { return p != nullptr && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Validates sizes shared by sfa_fwd / sfa_bwd and builds the virtual-problem geometry.
+bool use_mma_kernels();
+
 hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, int window,
                       SfaGeom* g) {
   if (B <= 0 || L <= 0 || n <= 0 || Hq <= 0 || Hkv <= 0 || Dh <= 0) return HD_ERR_INVALID_ARG;
   if (Hq % Hkv != 0) return HD_ERR_INVALID_ARG;
-  if (mode != SFA_WITHIN && mode != SFA_CROSS && mode != SFA_LOCAL) return HD_ERR_INVALID_ARG;
+  if (mode != SFA_WITHIN && mode != SFA_CROSS && mode != SFA_LOCAL && mode != SFA_WITHIN_NAIVE)
+    return HD_ERR_INVALID_ARG;
   if (mode == SFA_LOCAL && window <= 0) return HD_ERR_INVALID_ARG;
   if (Dh != 64 && Dh != 128 && Dh != 256) return HD_ERR_UNSUPPORTED;
+  // the naive schedule exists on the head-dim-128 tcgen05 kernels only
+  if (mode == SFA_WITHIN_NAIVE && (Dh != 128 || use_mma_kernels())) return HD_ERR_UNSUPPORTED;
   const long long nL = (long long)n * L;
   // Every row index, head product and tile count must fit the kernels' int math.
   if (nL > (1LL << 30) || (long long)B * nL * Hq > (1LL << 31) / 2) return HD_ERR_UNSUPPORTED;
@@ -73,12 +78,13 @@ hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t m
     g->ns = n;
     g->rs = n;
     g->window = 0;
-  } else {
+  } else {  // CROSS, LOCAL, and the naive WITHIN schedule
     g->Lv = (int)nL;
     g->ns = 1;
     g->rs = 1;
     g->window = mode == SFA_LOCAL ? window : 0;
   }
+  g->smod = mode == SFA_WITHIN_NAIVE ? n : 0;
   // queries are the key rows themselves
   g->Lq = g->Lv;
   g->qstep = 1;
@@ -94,6 +100,7 @@ hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t m
 // the loss reads, Eq. 2) in dense [B][L] tensors against the keys of the layer's mask.
 hd_status_t make_final_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, int window,
                             SfaGeom* g) {
+  if (mode == SFA_WITHIN_NAIVE) return HD_ERR_UNSUPPORTED;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, g);
   if (st != HD_OK) return st;
   g->Lq = L;

@@ -478,7 +478,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       // window edge at or above the tile's first key, ragged tiles
       const bool win_edge =
           WIN ? (qm + BQ - 1) * G.qstep + G.qoff - G.window >= n0 : G.window > 0;
-      if ((qm * G.qstep + G.qoff < n0 + BK) || win_edge || (n0 + BK > G.Lv) || (qm + BQ > G.Lq)) {
+      if ((qm * G.qstep + G.qoff < n0 + BK) || win_edge || (n0 + BK > G.Lv) || (qm + BQ > G.Lq) || G.smod > 1) {
         // key row kr sees the queries q in [vis_lo, vis_hi): q*qstep + qoff >= kr
         // (causal), q < Lq, and for LOCAL q*qstep + qoff < kr + window (an empty range
         // when kr itself is past Lv)
@@ -493,6 +493,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
 #pragma unroll
         for (int i = 0; i < 64; ++i)
           if (qb + i < vis_lo || qb + i >= vis_hi) w[i] = __float_as_uint(-INFINITY);
+        if (G.smod > 1) {  // the naive intra-stream schedule (CROSS rows: query row = key row)
+          int k = (qb - kr) % G.smod;  // (query row - key row) mod smod, stepped along the columns
+          if (k < 0) k += G.smod;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) {
+            if (k != 0) w[i] = __float_as_uint(-INFINITY);
+            k = k + 1 == G.smod ? 0 : k + 1;
+          }
+        }
       }
     };
     auto d_values = [&](uint32_t* w, const float* src) {  // dP'^T: -delta

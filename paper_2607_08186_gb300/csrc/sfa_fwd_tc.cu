@@ -70,7 +70,10 @@ HD_DEVINLINE void tile_range(const SfaGeom& G, int m0, int& lo, int& hi) {
 }
 
 // TMEM columns: S_g at g*128 (P_g packed bf16 over its first 64 columns), O_g at 256 + g*DH.
-template <int DH>
+// NAIVE: the naive intra-stream schedule (G.smod > 1): every tile is masked, a pair
+// also needing key row = query row (mod smod); its own instantiation, so the other
+// modes' softmax carries none of that code.
+template <int DH, bool NAIVE>
 __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant__ Params P) {
   extern __shared__ uint8_t smem_raw[];
   Smem<DH>& sm = *reinterpret_cast<Smem<DH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -241,7 +244,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
       // or below the last query's window edge, and the ragged last tile
       const bool need_mask = (j + 1) * BN - 1 > rq0 || (G.window > 0 && j * BN <= rq1 - G.window) ||
                              (j + 1) * BN > G.Lv;
-      if (need_mask) {
+      if constexpr (NAIVE) {
+        // causal (no window in this schedule) and k = (rq - key row) mod smod == 0,
+        // k stepped down the tile's columns
+        int k = (rq - j * BN) % G.smod;
+        if (k < 0) k += G.smod;
+#pragma unroll
+        for (int e = 0; e < BN; ++e) {
+          if (k != 0 || j * BN + e > rq || j * BN + e >= G.Lv) x[e] = -INFINITY;
+          k = k == 0 ? G.smod - 1 : k - 1;
+        }
+      } else if (need_mask) {
 #pragma unroll
         for (int e = 0; e < BN; ++e)
           if (!visible(rq, j * BN + e, G.Lv, G.window)) x[e] = -INFINITY;
@@ -335,14 +348,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
 }  // namespace tcfwd
 
 // --------------------------------------------------------------------- host
-template <int DH>
+template <int DH, bool NAIVE>
 static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   const int smem = (int)sizeof(tcfwd::Smem<DH>) + 1024;
-  cudaError_t e = cudaFuncSetAttribute(tcfwd::fwd_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e =
+      cudaFuncSetAttribute(tcfwd::fwd_kernel<DH, NAIVE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const unsigned grid = (unsigned)((p.g.Lq + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM)) *
                         (unsigned)(p.g.Hq * p.g.q_ns * p.g.B);
-  tcfwd::fwd_kernel<DH><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
+  tcfwd::fwd_kernel<DH, NAIVE><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }
 
@@ -358,7 +372,8 @@ cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void*
   p.g = g;
   p.scale_log2 = scale * tcfwd::kLog2e;
   p.status = status;
-  return Dh == 64 ? tc_fwd_impl<64>(p, st) : tc_fwd_impl<128>(p, st);
+  if (Dh == 64) return tc_fwd_impl<64, false>(p, st);
+  return g.smod > 1 ? tc_fwd_impl<128, true>(p, st) : tc_fwd_impl<128, false>(p, st);
 }
 
 }  // namespace hdsfa

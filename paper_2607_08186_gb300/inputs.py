@@ -13,7 +13,7 @@ from dataclasses import dataclass
 
 import torch
 
-WITHIN, CROSS, LOCAL = 0, 1, 2
+WITHIN, CROSS, LOCAL, WITHIN_NAIVE = 0, 1, 2, 3
 
 
 @dataclass(frozen=True)

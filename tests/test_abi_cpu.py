@@ -65,6 +65,22 @@ def test_fwd_validation(lib):
     assert _fwd(lib, Dh=32) == 2
 
 
+def test_naive_within_mode_validation(lib):
+    # the naive intra-stream schedule runs on the head-dim-128 tcgen05 kernels only, and
+    # takes the CROSS problem's workspace; final-stream and decode calls reject it
+    P, Z, F = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_float
+    assert _fwd(lib, mode=3, Dh=64) == 2
+    assert _fwd(lib, mode=3, Dh=256) == 2
+    assert _fwd(lib, mode=3, Dh=128, ptr=FAKE + 8) == 1  # misaligned: rejected before any launch
+    assert binding.sfa_bwd_workspace_bytes(1, 100, 4, 8, 2, 128, 3) == binding.sfa_bwd_workspace_bytes(
+        1, 100, 4, 8, 2, 128, 1)
+    assert binding.sfa_bwd_workspace_bytes(1, 100, 4, 8, 2, 64, 3) == 0
+    assert lib.sfa_bwd_final_workspace_bytes(1, 64, 4, 8, 2, 128, 3) == 0
+    assert lib.sfa_fwd_final(P(FAKE), P(FAKE), P(FAKE), P(FAKE), P(FAKE), 1, 64, 4, 8, 2, 128, F(0.0), 3, 0,
+                             None, None) == 2
+    assert binding.sfa_decode_workspace_bytes(1, 64, 4, 8, 2, 128, 3) == 0
+
+
 def test_bwd_workspace_size(lib):
     B, L, n, Hq, Hkv, Dh = 1, 100, 4, 8, 2, 128
     ws = binding.sfa_bwd_workspace_bytes(B, L, n, Hq, Hkv, Dh, 0)

@@ -11,7 +11,7 @@ import torch
 
 import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
-from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, WITHIN
+from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, WITHIN, WITHIN_NAIVE
 
 from parity import (assert_fwd_close, assert_grads_close, gpu_fwd, gpu_fwd_bwd, group_slices,
                     max_abs, sample_rows, TOL_LSE, TOL_O)
@@ -28,9 +28,10 @@ def _built():
 def _full_case(s: AttnShape, mode, seed, window=0, scale=0.0):
     q, k, v, do = inputs.attn_inputs(s, seed=seed)
     o, lse, dq, dk, dv = gpu_fwd_bwd(q, k, v, do, s.n, mode, scale, window)
-    o_ref, lse_ref = oracle.sfa_fwd(q, k, v, s.n, mode, scale or None, window)
+    om = WITHIN if mode == WITHIN_NAIVE else mode  # the naive schedule computes the WITHIN result
+    o_ref, lse_ref = oracle.sfa_fwd(q, k, v, s.n, om, scale or None, window)
     assert_fwd_close(o, lse, o_ref, lse_ref)
-    dq_r, dk_r, dv_r = oracle.sfa_bwd(q, k, v, do, s.n, mode, scale or None, window)
+    dq_r, dk_r, dv_r = oracle.sfa_bwd(q, k, v, do, s.n, om, scale or None, window)
     assert_grads_close([("dq", dq, dq_r), ("dk", dk, dk_r), ("dv", dv, dv_r)])
 
 
@@ -78,6 +79,14 @@ def test_head_dim_256_many_key_tiles(mode, window):
     # 1200 positions: up to 10 key tiles per query tile, so the head-dim-256 forward's
     # five-slot K/V ring wraps several times; ragged last tiles (1200 = 9*128 + 48)
     _full_case(AttnShape(1, 300, 4, 4, 2, 256), mode, seed=33, window=window)
+
+
+@pytest.mark.parametrize("shape", [(1, 100, 1, 4, 2, 128), (1, 130, 4, 4, 1, 128), (2, 77, 3, 4, 2, 128),
+                                   (1, 70, 8, 2, 2, 128)])
+def test_naive_within_schedule(shape):
+    # WITHIN's mask applied per pair over the full causal tile schedule of nL positions
+    # (no stream-tile skipping): the WITHIN oracle's result, forward and backward
+    _full_case(AttnShape(*shape), WITHIN_NAIVE, seed=61 + sum(shape))
 
 
 @pytest.mark.parametrize("window", [1, 50, 200])
@@ -147,6 +156,8 @@ def test_prep_halves_with_the_clear_on_a_side_stream(mode):
 def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
     q, k, v, do = inputs.attn_inputs(s, seed=seed)
     o, lse, dq, dk, dv = gpu_fwd_bwd(q, k, v, do, s.n, mode)
+    if mode == WITHIN_NAIVE:  # checked against the WITHIN oracle
+        mode = WITHIN
     grp = s.Hq // s.Hkv
     edges = [0, 1, 63, 64, 127, 128, s.nL // 2, s.nL - 129, s.nL - 2, s.nL - 1]
     rows = sample_rows(s.B, s.Hq, s.nL, n_rows, seed, edges)
@@ -176,7 +187,7 @@ def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
     assert_grads_close([("dk rows", dk[0, ps, g], dk_r), ("dv rows", dv[0, ps, g], dv_r)])
 
 
-@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+@pytest.mark.parametrize("mode", [WITHIN, CROSS, WITHIN_NAIVE])
 def test_qwen3_8b_class_layer(mode):
     # B=1, L=4096, n=4 (16384 positions), Hq=32, Hkv=8, Dh=128
     _sampled_parity(inputs.SHAPES["qwen3_8b_n4"], mode, seed=1)
