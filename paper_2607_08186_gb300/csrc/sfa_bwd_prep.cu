@@ -15,10 +15,15 @@ namespace hdsfa {
 
 typedef __nv_bfloat16 bf16;
 
-// One warp takes RPW consecutive (b, p, h) rows: DH/8 lanes per row (16 bytes of O and
-// of dO each), 32*8/DH rows side by side, ITER such row groups with every load issued
-// before the first dot product, so each warp keeps several KB in flight.  With ZERO the
-// warp then zeroes the same rows of the fp32 dQ accumulator (contiguous, 16-byte stores).
+// One warp takes the 8 consecutive rows r0..r0+7 of one (b, head h, stream s) problem
+// (positions p = r*ns + s): each row's O and dO are DH*2 contiguous bytes (DH/8 lanes,
+// 16 bytes each, 32*8/DH rows per load instruction, every load issued before the
+// first dot product); the rows' LSE values lie within 8*ns floats and their row terms
+// are 8 consecutive floats of the stream-major arrays, so lanes 0..7 load the LSE
+// together and, after the dot products are gathered to them, store both row terms
+// as one 32-byte run each.  Warps are ordered head-fastest, so a CTA's eight warps
+// read the eight heads' rows that share positions (adjacent in memory).  With ZERO the
+// warp then zeroes its rows of the fp32 dQ accumulator.
 template <int DH, bool ZERO>
 __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restrict__ o,
                                                            const bf16* __restrict__ dout,
@@ -26,52 +31,68 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
                                                            float* __restrict__ lse2_t,
                                                            float* __restrict__ delta_t,
                                                            float* __restrict__ dq_acc, SfaGeom g) {
-  constexpr int LPR = DH / 8;        // lanes per row
-  constexpr int RPG = 32 / LPR;      // rows per group of the warp
-  constexpr int ITER = 4;            // row groups per warp
-  constexpr int RPW = RPG * ITER;    // rows per warp
+  constexpr int LPR = DH / 8;      // lanes per row
+  constexpr int RPG = 32 / LPR;    // rows per load instruction
+  constexpr int RPW = 8;           // rows per warp
+  constexpr int ITER = RPW / RPG;  // load instructions per tensor
   const int lane = threadIdx.x & 31, sub = lane / LPR, l = lane % LPR;
-  // row indices fit 32 bits (the host caps B*nL*Hq below 2^30): 32-bit index math, whose
-  // divisions cost a fraction of 64-bit ones
-  const long long nrows = (long long)g.B * g.nL * g.Hq;
-  const long long row0 = (((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5) * RPW;
-  if (row0 >= nrows) return;
+  // warp -> (b, s, r-block, h), h fastest; 32-bit index math (the host caps B*nL*Hq
+  // below 2^30)
+  const unsigned Hq = (unsigned)g.Hq, ns = (unsigned)g.ns, Lv = (unsigned)g.Lv, nL = (unsigned)g.nL;
+  const unsigned nrb = (Lv + RPW - 1) / RPW;
+  const unsigned w = (unsigned)(((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  if ((long long)w >= (long long)g.B * ns * nrb * Hq) return;
+  const unsigned h = w % Hq, w1 = w / Hq, rb = w1 % nrb, w2 = w1 / nrb, s = w2 % ns, b = w2 / ns;
+  const unsigned r0 = rb * RPW;
   uint4 xo[ITER], xd[ITER];
 #pragma unroll
   for (int i = 0; i < ITER; ++i) {
-    const long long row = row0 + i * RPG + sub;
-    if (row < nrows) {
+    const unsigned r = r0 + i * RPG + sub;
+    xo[i] = make_uint4(0, 0, 0, 0);
+    xd[i] = make_uint4(0, 0, 0, 0);
+    if (r < Lv) {
+      const long long row = ((long long)b * nL + (long long)r * ns + s) * Hq + h;
       xo[i] = *reinterpret_cast<const uint4*>(o + row * DH + l * 8);
       xd[i] = *reinterpret_cast<const uint4*>(dout + row * DH + l * 8);
-    } else {
-      xo[i] = make_uint4(0, 0, 0, 0);
-      xd[i] = make_uint4(0, 0, 0, 0);
     }
   }
-  const int Lvp = row_terms_pitch(g.Lv);
+  const long long bh = (long long)b * Hq + h;
+  const bool mine = lane < RPW && r0 + lane < Lv;  // lane j: row r0 + j's LSE and row terms
+  const float lv = mine ? lse[bh * nL + (long long)(r0 + lane) * ns + s] : 0.f;
+  float acc[ITER];
 #pragma unroll
   for (int i = 0; i < ITER; ++i) {
     const bf16* xa = reinterpret_cast<const bf16*>(&xo[i]);
     const bf16* ya = reinterpret_cast<const bf16*>(&xd[i]);
-    float acc = 0.f;
+    float a = 0.f;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) acc += __bfloat162float(xa[e]) * __bfloat162float(ya[e]);
+    for (int e = 0; e < 8; ++e) a += __bfloat162float(xa[e]) * __bfloat162float(ya[e]);
 #pragma unroll
-    for (int off = LPR / 2; off; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-    const long long row = row0 + i * RPG + sub;
-    if (l == 0 && row < nrows) {
-      const unsigned ur = (unsigned)row, Hq = (unsigned)g.Hq, nL = (unsigned)g.nL, ns = (unsigned)g.ns;
-      const unsigned bp = ur / Hq, h = ur - bp * Hq, b = bp / nL, p = bp - b * nL;
-      const unsigned r = p / ns, s = p - r * ns;
-      const long long t = (((long long)b * Hq + h) * ns + s) * Lvp + r;
-      delta_t[t] = -acc;
-      lse2_t[t] = -lse[((long long)b * Hq + h) * nL + p] * 1.4426950408889634f;
-    }
+    for (int off = LPR / 2; off; off >>= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
+    acc[i] = a;  // row r0 + i*RPG + sub, in every lane of its group
   }
-  if (ZERO) {  // zero dQ accumulator rows [row0, row0 + RPW): RPW * DH floats, contiguous
-    const long long nz = (min(nrows, row0 + RPW) - row0) * DH / 4;
-    float4* dz = reinterpret_cast<float4*>(dq_acc + row0 * DH);
-    for (long long c = lane; c < nz; c += 32) dz[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+  float dl = 0.f;  // lane j < 8: the dot product of row r0 + j
+#pragma unroll
+  for (int i = 0; i < ITER; ++i)
+#pragma unroll
+    for (int sb = 0; sb < RPG; ++sb) {
+      const float v = __shfl_sync(0xffffffffu, acc[i], sb * LPR);
+      if (lane == i * RPG + sb) dl = v;
+    }
+  if (mine) {
+    const long long t = (bh * ns + s) * row_terms_pitch(g.Lv) + r0 + lane;
+    delta_t[t] = -dl;
+    lse2_t[t] = -lv * 1.4426950408889634f;
+  }
+  if (ZERO) {  // this warp's rows of the dQ accumulator, DH contiguous floats each
+#pragma unroll
+    for (int j = 0; j < RPW; ++j) {
+      const unsigned r = r0 + j;
+      if (r < Lv) {
+        float4* dz = reinterpret_cast<float4*>(dq_acc + (((long long)b * nL + (long long)r * ns + s) * Hq + h) * DH);
+        for (int c = lane; c < DH / 4; c += 32) dz[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
   }
 }
 
@@ -108,9 +129,7 @@ __global__ void __launch_bounds__(256) sfa_bwd_finalize_kernel(const float* __re
 cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
                                 float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
                                 cudaStream_t st, bool zero) {
-  const long long rows = (long long)g.B * g.nL * g.Hq;
-  const long long rpw = 4LL * (32 / (Dh / 8));  // rows per warp (ITER * rows per group)
-  const long long warps = (rows + rpw - 1) / rpw;
+  const long long warps = (long long)g.B * g.ns * ((g.Lv + 7) / 8) * g.Hq;  // 8 rows of one problem each
   const unsigned blocks = (unsigned)((warps * 32 + 255) / 256);
   const bf16 *ob = (const bf16*)o, *db = (const bf16*)dout;
   if (Dh == 256) {
