@@ -5,6 +5,7 @@
 #include <string.h>
 
 #include "common.cuh"
+#include "decode_plan.cuh"
 
 namespace hdsfa {
 cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L,
@@ -16,12 +17,6 @@ cudaError_t launch_expand_bwd_apply(const void* dx, float* de, int B, int L, int
                                     cudaStream_t st);
 cudaError_t launch_select_final(const void* x, void* y, int B, int L, int n, int D, cudaStream_t st);
 cudaError_t launch_select_final_bwd(const void* dy, void* dx, int B, int L, int n, int D, cudaStream_t st);
-struct DecodePlan {
-  int G, M, ngroups, nsplit, chunk;
-  size_t part_o_bytes, part_ml_bytes;
-};
-DecodePlan decode_plan(int B, int maxT, int n, int Hq, int Hkv, int Dh, int mode, int window);
-size_t decode_ws_bytes(const DecodePlan& p);
 cudaError_t launch_sfa_decode(const void* q, const void* kc, const void* vc, const int32_t* lens, void* o,
                               float* lse, int B, int maxT, int Lcap, int n, int Hq, int Hkv, int Dh, float scale,
                               int mode, int window, void* ws, int32_t* status, cudaStream_t st);

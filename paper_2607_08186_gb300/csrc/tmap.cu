@@ -36,4 +36,20 @@ bool make_rows_tmap(CUtensorMap* m, const void* base, const SfaGeom& g, int H, i
   return r == CUDA_SUCCESS;
 }
 
+// Tensor map over the decoding step's queries q [B][n][Hq][Dh] seen as {Dh, Hq, n, B};
+// box = 64 columns x G heads x n streams of one sequence, so one load per 64 columns
+// brings the n*G query rows of a K/V head's group, row s*G + (head - first head).
+bool make_qgroup_tmap(CUtensorMap* m, const void* base, int B, int n, int Hq, int Dh, int G) {
+  auto enc = tmap_encoder();
+  if (enc == nullptr) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)Dh, (cuuint64_t)Hq, (cuuint64_t)n, (cuuint64_t)B};
+  cuuint64_t strides[3] = {(cuuint64_t)Dh * 2, (cuuint64_t)Hq * Dh * 2, (cuuint64_t)n * Hq * Dh * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)n, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 }  // namespace hdsfa

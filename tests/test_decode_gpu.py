@@ -72,10 +72,11 @@ def test_shapes_ragged(mode, w, n, Hq, Hkv):
 
 
 @pytest.mark.parametrize("mode,w", [(WITHIN, 0), (CROSS, 0), (LOCAL, 1), (LOCAL, 100)])
-@pytest.mark.parametrize("n,Hq,Hkv", [(4, 24, 2), (4, 4, 1), (3, 6, 2)])
+@pytest.mark.parametrize("n,Hq,Hkv", [(4, 24, 2), (4, 4, 1), (3, 6, 2), (8, 32, 2), (8, 64, 2)])
 def test_head_dim_256_ragged(mode, w, n, Hq, Hkv):
-    # head dim 256 (Table 6's 80B heads: 24 query over 2 K/V heads, 48 query rows per K/V
-    # head in two row groups), one m16 tile, and 9 rows; lengths 1, 129 and the capacity
+    # head dim 256: Table 6's 80B heads (24 query over 2 K/V heads: 48 query rows per K/V
+    # head), 16, 9 and exactly 128 rows (one tcgen05 tile, rows padded to 128), and 256 rows
+    # (the mma.sync kernel's row groups); lengths 1, 129 and the capacity
     Lcap = 300
     q, kc, vc = _case(3, Lcap, n, Hq, Hkv, 256, 40 + n + Hq)
     _check(q, kc, vc, torch.tensor([Lcap, 1, 129], dtype=torch.int32), n, mode, w)
