@@ -454,33 +454,38 @@ def final_pairs(L: int, n: int, mode: int, window: int = 0) -> int:
 
 def measure_final_layer(dev, bf16_peak: float, iters: int = 5):
     """Final-stream-only layer (Sec. 3.1 KV-mirror layers: the L final-stream queries against
-    all nL keys), Qwen3-8B-class heads, L=4096, n=4: fwd and bwd TFLOP/s over visible pairs."""
+    all nL keys), L=4096, n=4, with Qwen3-8B-class heads (Hq=32, Hkv=8, Dh=128) and the 80B
+    configuration's heads (Hq=24, Hkv=2, Dh=256, Table 6): fwd and bwd TFLOP/s over
+    visible pairs."""
     from paper_2607_08186_gb300 import binding
-    B, L, n, Hq, Hkv, Dh = 1, 4096, 4, 32, 8, 128
+    B, L, n = 1, 4096, 4
     g = torch.Generator(device=dev)
     g.manual_seed(51)
 
     def rnd(*shape):
         return torch.randn(*shape, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
 
-    q, do = rnd(B, L, Hq, Dh), rnd(B, L, Hq, Dh)
-    k, v = rnd(B, n * L, Hkv, Dh), rnd(B, n * L, Hkv, Dh)
-    o, lse = torch.empty_like(q), torch.empty(B, Hq, L, dtype=torch.float32, device=dev)
-    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
-    out = {"workload": f"final-stream layer B={B} L={L} n={n} ({n * L} key positions) Hq={Hq} Hkv={Hkv} Dh={Dh}"}
-    for mode in (WITHIN, CROSS):
-        ws = torch.empty(binding.sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
-                         device=dev)
-        tf = time_op(lambda k_: binding.sfa_fwd_final(q, k, v, o, lse, mode), 1, iters=iters)
-        tb = time_op(lambda k_: binding.sfa_bwd_final(q, k, v, o, lse, do, dq, dk, dv, mode, ws), 1, iters=iters)
-        pairs = final_pairs(L, n, mode) * Hq * B
-        out[MODE_NAME[mode]] = {"fwd_ms": tf * 1e3, "bwd_ms": tb * 1e3,
-                                "fwd_tflops": FWD_FLOP * Dh * pairs / tf / 1e12,
-                                "bwd_tflops": BWD_FLOP * Dh * pairs / tb / 1e12,
-                                "fwd_frac": FWD_FLOP * Dh * pairs / tf / 1e12 / bf16_peak,
-                                "bwd_frac": BWD_FLOP * Dh * pairs / tb / 1e12 / bf16_peak}
-    del q, do, k, v, o, lse, dq, dk, dv
-    torch.cuda.empty_cache()
+    out = {"workload": f"final-stream layer B={B} L={L} n={n} ({n * L} key positions)"}
+    for name, Hq, Hkv, Dh in (("qwen3_8b", 32, 8, 128), ("80b", 24, 2, 256)):
+        q, do = rnd(B, L, Hq, Dh), rnd(B, L, Hq, Dh)
+        k, v = rnd(B, n * L, Hkv, Dh), rnd(B, n * L, Hkv, Dh)
+        o, lse = torch.empty_like(q), torch.empty(B, Hq, L, dtype=torch.float32, device=dev)
+        dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+        res = {"heads": f"Hq={Hq} Hkv={Hkv} Dh={Dh}"}
+        for mode in (WITHIN, CROSS):
+            ws = torch.empty(binding.sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
+                             device=dev)
+            tf = time_op(lambda k_: binding.sfa_fwd_final(q, k, v, o, lse, mode), 1, iters=iters)
+            tb = time_op(lambda k_: binding.sfa_bwd_final(q, k, v, o, lse, do, dq, dk, dv, mode, ws), 1, iters=iters)
+            pairs = final_pairs(L, n, mode) * Hq * B
+            res[MODE_NAME[mode]] = {"fwd_ms": tf * 1e3, "bwd_ms": tb * 1e3,
+                                    "fwd_tflops": FWD_FLOP * Dh * pairs / tf / 1e12,
+                                    "bwd_tflops": BWD_FLOP * Dh * pairs / tb / 1e12,
+                                    "fwd_frac": FWD_FLOP * Dh * pairs / tf / 1e12 / bf16_peak,
+                                    "bwd_frac": BWD_FLOP * Dh * pairs / tb / 1e12 / bf16_peak}
+        out[name] = res
+        del q, do, k, v, o, lse, dq, dk, dv, ws
+        torch.cuda.empty_cache()
     return out
 
 

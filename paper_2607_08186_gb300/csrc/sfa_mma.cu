@@ -41,7 +41,6 @@ struct MmaBwdArgs {
   SfaGeom g;
   float scale;
   float scale_log2;
-  int d0;  // first head-dim column of the dK / dV / dQ slice this launch writes
 };
 
 // rows [r0, r0 + ROWS) of a [*][DH] row set (row stride rstride elements) -> swizzled smem.
@@ -247,9 +246,10 @@ __global__ void __launch_bounds__(NT) sfa_fwd_mma_kernel(MmaFwdArgs a) {
 // registers while looping over the group's query heads and the query tiles that
 // can see tile j; dQ contributions go to the fp32 accumulator with atomics.
 // Warp w owns key rows [16w, 16w + 16) of the tile for S^T, dP^T, dK, dV.
-// DO: the head-dim columns of dK, dV, dQ one launch accumulates (starting at a.d0);
-// S^T and dP^T always take the full head dim.  DO = DH in one launch, or two launches
-// of DO = DH / 2 at head dim 256 (whose dK and dV would not fit the registers at once).
+// DO: the head-dim columns of dK, dV, dQ one CTA accumulates (starting at d0); S^T and
+// dP^T always take the full head dim.  DO = DH, or DO = DH / 2 at head dim 256 (whose
+// dK and dV would not fit the registers at once), the two slices of a key tile being
+// separate CTAs of one launch.
 template <int DH, int DO>
 __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem_raw[];
@@ -267,7 +267,10 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   const int ntile = (G.Lq + BM - 1) / BM;
   const int j = blockIdx.x;  // key tile; tile 0 sees the most query tiles, so it starts first
   const int n0 = j * BN;
-  const int kvh = blockIdx.y / G.q_ns, s = blockIdx.y % G.q_ns, b = blockIdx.z;
+  const int kvh = blockIdx.y / G.q_ns, s = blockIdx.y % G.q_ns;
+  // blockIdx.z: batch and head-dim slice (the DO columns of dK, dV, dQ from d0 this CTA
+  // writes; the slices of one key tile run side by side)
+  const int b = blockIdx.z / (DH / DO), d0 = (blockIdx.z % (DH / DO)) * DO;
   const int sk = s + G.kv_s0;  // stream of the key problem
   const int grp = G.Hq / G.Hkv;
   // query tiles that can see a key of this tile: query row r stands at key row
@@ -390,7 +393,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
         const int qrow = half * 32 + kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
         for (int dp = 0; dp < DO / 16; ++dp) {
-          const int dcol = a.d0 + dp * 16 + (lane >> 4) * 8;
+          const int dcol = d0 + dp * 16 + (lane >> 4) * 8;
           uint32_t b0, b1, b2, b3;
           ldsm_x4_t(smem_u32(cdO + swz<DH>(qrow, dcol)), b0, b1, b2, b3);
           mma_bf16_16816(dV[2 * dp], pa, b0, b1);
@@ -428,7 +431,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
           for (int dp = 0; dp < DO / 32; ++dp) {
             uint32_t b0, b1, b2, b3;
             ldsm_x4_t(smem_u32(sK + swz<DH>(kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8,
-                                            a.d0 + dh * (DO / 2) + dp * 16 + (lane >> 4) * 8)),
+                                            d0 + dh * (DO / 2) + dp * 16 + (lane >> 4) * 8)),
                       b0, b1, b2, b3);
             mma_bf16_16816(qacc[2 * dp], aa, b0, b1);
             mma_bf16_16816(qacc[2 * dp + 1], aa, b2, b3);
@@ -436,7 +439,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
         }
 #pragma unroll
         for (int i = 0; i < DO / 16; ++i) {
-          const int col = a.d0 + dh * (DO / 2) + i * 8 + 2 * t4;
+          const int col = d0 + dh * (DO / 2) + i * 8 + 2 * t4;
           if (qa < G.Lq)
             atomicAdd(reinterpret_cast<float2*>(dqb + (long long)qa * q_rs + col),
                       make_float2(qacc[i][0], qacc[i][1]));
@@ -459,7 +462,7 @@ __global__ void __launch_bounds__(NT, 1) sfa_bwd_mma_kernel(MmaBwdArgs a) {
   const int kr = n0 + warp * 16 + g4;
 #pragma unroll
   for (int i = 0; i < DO / 8; ++i) {
-    const int col = a.d0 + i * 8 + 2 * t4;
+    const int col = d0 + i * 8 + 2 * t4;
     if (kr < G.Lv) {
       *reinterpret_cast<uint32_t*>(dkb + (long long)kr * kv_rs + col) =
           pack_bf16(dK[i][0] * a.scale, dK[i][1] * a.scale);
@@ -500,14 +503,10 @@ static cudaError_t bwd_impl(MmaBwdArgs a, cudaStream_t st) {
   const int smem = (2 * BN * DH + 4 * BM * DH + BN * BM) * (int)sizeof(bf16) + 4 * BM * (int)sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(sfa_bwd_mma_kernel<DH, DO>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.q_ns, g.B);
-  for (int d0 = 0; d0 < DH; d0 += DO) {  // one launch per output slice
-    a.d0 = d0;
-    sfa_bwd_mma_kernel<DH, DO><<<grid, NT, smem, st>>>(a);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-  }
-  return cudaSuccess;
+  // the DH / DO head-dim slices of every key tile in one launch
+  dim3 grid((g.Lv + BN - 1) / BN, g.Hkv * g.q_ns, g.B * (DH / DO));
+  sfa_bwd_mma_kernel<DH, DO><<<grid, NT, smem, st>>>(a);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const void* dout,
@@ -515,7 +514,7 @@ cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v,
                                     float* dq_ws, const SfaGeom& g, int Dh, float scale,
                                     cudaStream_t st) {
   MmaBwdArgs a{(const bf16*)q, (const bf16*)k, (const bf16*)v, (const bf16*)dout, lse2_ws, delta_ws,
-               dq_ws, (bf16*)dk, (bf16*)dv, g, scale, scale * kLog2e, 0};
+               dq_ws, (bf16*)dk, (bf16*)dv, g, scale, scale * kLog2e};
   if (Dh == 64) return bwd_impl<64, 64>(a, st);
   if (Dh == 256) return bwd_impl<256, 128>(a, st);
   return bwd_impl<128, 128>(a, st);
