@@ -299,7 +299,7 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
   // head dim 128 runs on the tcgen05 kernel; head dims 64 and 256 on the mma.sync kernel
-  // (at 256 in two launches, one per half of the dK / dV / dQ columns)
+  // (at 256 as two CTAs per key tile, one per half of the dK / dV / dQ columns)
   if (Dh == 128 && !use_mma_kernels())
     return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
                                                      scale, dev_status, stream));
