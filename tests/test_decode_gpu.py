@@ -82,8 +82,9 @@ def test_head_dim_256_ragged(mode, w, n, Hq, Hkv):
     _check(q, kc, vc, torch.tensor([Lcap, 1, 129], dtype=torch.int32), n, mode, w)
 
 
-def test_max_tokens_below_capacity():
-    q, kc, vc = _case(2, 500, 4, 8, 2, 128, 5)
+@pytest.mark.parametrize("Hq,Hkv,Dh", [(8, 2, 128), (24, 2, 256)])
+def test_max_tokens_below_capacity(Hq, Hkv, Dh):
+    q, kc, vc = _case(2, 500, 4, Hq, Hkv, Dh, 5)
     _check(q, kc, vc, torch.tensor([200, 77], dtype=torch.int32), 4, CROSS, max_tokens=200)
 
 
@@ -168,11 +169,13 @@ def test_append_then_decode_equals_forward_rows(Hq, Hkv, Dh):
         assert float((got_l - lse_r).abs().max()) <= 1e-3
 
 
-def test_serving_loop_in_a_cuda_graph():
+@pytest.mark.parametrize("Hq,Hkv,Dh", [(8, 2, 128), (24, 2, 256)])
+def test_serving_loop_in_a_cuda_graph(Hq, Hkv, Dh):
     # one step of a serving loop (append the new token's n K/V rows, then an intra-stream
     # and a cross-stream decode over the cache) captured once as a CUDA graph and replayed
     # while the sequences grow; every replay equals the oracle on the cache as it stands
-    B, n, Hq, Hkv, Dh, Lcap = 2, 4, 8, 2, 128, 64
+    # (head dim 256 with 24 over 2 heads: the tcgen05 decode kernel)
+    B, n, Lcap = 2, 4, 64
     lens0 = [20, 33]
     kc = torch.zeros(B, Lcap * n, Hkv, Dh, dtype=torch.bfloat16, device="cuda")
     vc = torch.zeros_like(kc)
