@@ -317,21 +317,23 @@ __global__ void __launch_bounds__(NT) decode_kernel(DecodeArgs a) {
   }
 }
 
-// CTA (K/V head x row group, sequence, 8-column slice); one warp per query row, its
-// lanes over the splits: the row's max and sum by warp reductions, then the slice of
-// O as the weighted sum of the splits' partial slices, written as bf16 (round to
-// nearest even); the first slice's CTA also writes the natural-log LSE.
+// CTA (K/V head x row group, sequence, 8-column slice x block of 8 rows); one warp per
+// query row, its lanes over the splits: the row's max and sum by warp reductions, then
+// the slice of O as the weighted sum of the splits' partial slices, written as bf16
+// (round to nearest even); the first slice's CTAs also write the natural-log LSE.
 template <int DH>
 __global__ void __launch_bounds__(256) combine_kernel(DecodeArgs a) {
-  const int g = blockIdx.x / a.ngroups, rg = blockIdx.x % a.ngroups, b = blockIdx.y, c8 = blockIdx.z;
+  const int g = blockIdx.x / a.ngroups, rg = blockIdx.x % a.ngroups, b = blockIdx.y;
+  const int c8 = blockIdx.z % (DH / 8), rb = blockIdx.z / (DH / 8);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rows = min(a.rg, a.M - rg * a.rg);
   const size_t pidx0 = (((size_t)b * a.Hkv + g) * a.ngroups + rg) * a.nsplit;
   grid_dep_wait();  // every partial of the decode kernel is written
   const int T = a.lens[b];
   const bool valid = T >= 1 && T <= a.maxT;
-  if (!valid && blockIdx.x == 0 && c8 == 0 && threadIdx.x == 0) set_status(a.status, HD_DEVBIT_INDEX);
-  for (int row = warp; row < rows; row += 8) {
+  if (!valid && blockIdx.x == 0 && blockIdx.z == 0 && threadIdx.x == 0) set_status(a.status, HD_DEVBIT_INDEX);
+  const int row = rb * 8 + warp;
+  if (row < rows) {
     float m = -INFINITY;
     for (int c = lane; c < a.nsplit; c += 32) m = fmaxf(m, a.part_ml[(pidx0 + c) * a.rg + row].x);
 #pragma unroll
@@ -785,7 +787,7 @@ static cudaError_t launch_decode_t(const dec::DecodeArgs& a, cudaStream_t st) {
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, decode_kernel<DH, MT>, a);
   if (e != cudaSuccess) return e;
-  cfg.gridDim = dim3(a.Hkv * a.ngroups, a.B, DH / 8);
+  cfg.gridDim = dim3(a.Hkv * a.ngroups, a.B, (DH / 8) * ((std::min(a.rg, a.M) + 7) / 8));
   cfg.blockDim = dim3(256);
   cfg.dynamicSmemBytes = 0;
   return cudaLaunchKernelEx(&cfg, combine_kernel<DH>, a);
@@ -822,7 +824,7 @@ static cudaError_t launch_decode_tc(const dec::DecodeArgs& a, cudaStream_t st) {
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, decode_tc_kernel, p);
   if (e != cudaSuccess) return e;
-  cfg.gridDim = dim3(a.Hkv, a.B, DH / 8);
+  cfg.gridDim = dim3(a.Hkv, a.B, (DH / 8) * ((std::min(a.rg, a.M) + 7) / 8));
   cfg.blockDim = dim3(256);
   cfg.dynamicSmemBytes = 0;
   return cudaLaunchKernelEx(&cfg, dec::combine_kernel<DH>, a);
