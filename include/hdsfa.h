@@ -294,6 +294,17 @@ hd_status_t sfa_bwd_noalloc(const void* q, const void* k, const void* v, const v
 /* Human-readable name of a status code (static string). */
 const char* hd_status_string(hd_status_t status);
 
+/*
+ * hd_selftest_bounded_wait -- diagnostic of the failure path shared by the tensor-core
+ * kernels (no counterpart in the paper).  Launches one warp that waits, with the same
+ * bounded mbarrier wait those kernels use, on a barrier nothing arrives on.  After the
+ * bound (about a second) the wait gives up: HD_DEVBIT_TIMEOUT is ORed into *dev_status
+ * and *dev_result is set to 0 (1 would mean the wait completed).  No fault, no trap: the
+ * kernel returns and the context stays usable.
+ *   dev_status, dev_result: device int32 words (dev_status may be NULL; dev_result not).
+ */
+hd_status_t hd_selftest_bounded_wait(int32_t* dev_status, int32_t* dev_result, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

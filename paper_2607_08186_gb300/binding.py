@@ -41,6 +41,8 @@ def lib():
                                    "paper_2607_08186_gb300.build.build() first")
             L = ctypes.CDLL(LIB_PATH)
             P, I, F, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+            L.hd_selftest_bounded_wait.restype = I
+            L.hd_selftest_bounded_wait.argtypes = [P, P, P]
             L.hd_expand_embed.restype = I
             L.hd_expand_embed.argtypes = [P, P, P, I, I, I, I, I, P, P]
             L.hd_expand_embed_bwd_workspace_bytes.restype = Z
@@ -93,6 +95,13 @@ def lib():
 
 def hd_status_string(code: int) -> str:
     return lib().hd_status_string(int(code)).decode()
+
+
+def hd_selftest_bounded_wait(dev_status, dev_result, stream=None):
+    """Diagnostic: one warp's bounded wait on a barrier nothing arrives on runs out
+    (about a second); HD_DEVBIT_TIMEOUT lands in dev_status, 0 in dev_result."""
+    _check(lib().hd_selftest_bounded_wait(_p(dev_status), _p(dev_result), _stream(stream)),
+           "hd_selftest_bounded_wait")
 
 
 def _p(t):

@@ -20,6 +20,7 @@ cudaError_t launch_select_final_bwd(const void* dy, void* dx, int B, int L, int 
 cudaError_t launch_sfa_decode(const void* q, const void* kc, const void* vc, const int32_t* lens, void* o,
                               float* lse, int B, int maxT, int Lcap, int n, int Hq, int Hkv, int Dh, float scale,
                               int mode, int window, void* ws, int32_t* status, cudaStream_t st);
+cudaError_t launch_bounded_wait_selftest(int32_t* status, int32_t* result, cudaStream_t st);
 cudaError_t launch_kv_append(const void* kn, const void* vn, void* kc, void* vc, const int32_t* lens, int B,
                              int Lcap, int n, int Hkv, int Dh, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
@@ -440,6 +441,12 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
   }
   if (e == cudaSuccess) e = hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, gq, Dh, scale, stream);
   return cuda_status(e);
+}
+
+hd_status_t hd_selftest_bounded_wait(int32_t* dev_status, int32_t* dev_result, cudaStream_t stream) {
+  if (dev_result == nullptr || (reinterpret_cast<uintptr_t>(dev_result) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  if (dev_status != nullptr && (reinterpret_cast<uintptr_t>(dev_status) & 3u) != 0) return HD_ERR_INVALID_ARG;
+  return cuda_status(hdsfa::launch_bounded_wait_selftest(dev_status, dev_result, stream));
 }
 
 const char* hd_status_string(hd_status_t s) {
