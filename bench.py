@@ -492,13 +492,14 @@ def measure_final_layer(dev, bf16_peak: float, iters: int = 5):
 def measure_decode(dev, hbm_peak: float, quick: bool = False):
     """Decoding step (Sec. 3.2), n=4: the new token's 4 positions against a context of T
     tokens (4T cached positions) for batch B, WITHIN and CROSS layers, with Qwen3-8B-class
-    heads (Hq=32, Hkv=8, Dh=128) and, unless quick, 80B-class heads (Hq=24, Hkv=2, Dh=256,
-    Table 6).  Algorithmic bytes: the visible cached K and V rows (B*T*n*Hkv*Dh*2 bytes
+    heads (Hq=32, Hkv=8, Dh=128) and, unless quick, the 80B configuration's heads (Hq=24,
+    Hkv=2, Dh=256) and the 617B configuration's (Hq=96, Hkv=8, Dh=128) of Table 6.  Algorithmic bytes: the visible cached K and V rows (B*T*n*Hkv*Dh*2 bytes
     each) plus q and o; rotating cache sets keep every call out of L2."""
     from paper_2607_08186_gb300 import binding
     n = 4
     heads = {"qwen3_8b": (32, 8, 128, [(1, 8192), (4, 8192), (16, 8192), (1, 32768), (16, 32768)]),
-             "80b": (24, 2, 256, [(1, 8192), (16, 8192), (1, 32768), (16, 32768)])}
+             "80b": (24, 2, 256, [(1, 8192), (16, 8192), (1, 32768), (16, 32768)]),
+             "617b": (96, 8, 128, [(1, 8192), (16, 8192)])}
     if quick:
         heads = {"qwen3_8b": (32, 8, 128, [(1, 8192), (16, 8192)])}
     res = {}

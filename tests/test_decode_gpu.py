@@ -62,10 +62,12 @@ def test_tiny(mode, w):
 
 
 @pytest.mark.parametrize("mode,w", [(WITHIN, 0), (CROSS, 0), (LOCAL, 1), (LOCAL, 100)])
-@pytest.mark.parametrize("n,Hq,Hkv", [(4, 32, 8), (8, 32, 8), (8, 64, 8), (1, 8, 8), (3, 6, 2)])
+@pytest.mark.parametrize("n,Hq,Hkv", [(4, 32, 8), (8, 32, 8), (8, 64, 8), (1, 8, 8), (3, 6, 2), (4, 96, 8),
+                                     (8, 128, 8)])
 def test_shapes_ragged(mode, w, n, Hq, Hkv):
-    # query rows per K/V head: 16 (one m16 tile), 32 (two), 64 (two CTAs per head),
-    # 1 and 9; lengths 1, 129 and the full capacity in one batch
+    # query rows per K/V head: 16 (one m16 tile), 32 (two), 64 and 128 (two and four CTAs
+    # per head), 48 (Table 6's 617B layout: 96 query over 8 K/V heads), 1 and 9; lengths
+    # 1, 129 and the full capacity in one batch
     Lcap = 300
     q, kc, vc = _case(3, Lcap, n, Hq, Hkv, 128, n + Hq)
     _check(q, kc, vc, torch.tensor([Lcap, 1, 129], dtype=torch.int32), n, mode, w)
@@ -123,6 +125,14 @@ def test_full_size_head_dim_256(mode):
     # shorter sequence; every output row checked against the oracle
     q, kc, vc = _case(2, 8192, 4, 24, 2, 256, 18)
     _check(q, kc, vc, torch.tensor([8192, 3001], dtype=torch.int32), 4, mode)
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_full_size_617b_heads(mode):
+    # the 617B configuration's head layout (96 query over 8 K/V heads, Dh=128: 48 query
+    # rows per K/V head, two row groups), n = 4, an 8192-token context, B = 2
+    q, kc, vc = _case(2, 8192, 4, 96, 8, 128, 28)
+    _check(q, kc, vc, torch.tensor([8192, 4321], dtype=torch.int32), 4, mode)
 
 
 def test_kv_append_bit_exact_and_flag():
