@@ -4,8 +4,9 @@
 One step = one pass of the hot path over one synthetic batch of the
 Qwen3-8B-class layer (B=1, L=4096 tokens, n=4 -> 16384 positions, Hq=32, Hkv=8,
 Dh=128, bf16, intra-stream / WITHIN mask):
-  expansion gather (4 tables of 151936 x 4096)  -> sfa_fwd -> sfa_bwd_prep
-  -> sfa_bwd_main -> sfa_bwd_finalize.
+  expansion gather (4 tables of 151936 x 4096)  -> sfa_fwd -> sfa_bwd_row_terms
+  -> sfa_bwd_main -> sfa_bwd_finalize, with sfa_bwd_clear on a side stream beside
+  the forward.
 Metric: attention FLOPs over visible pairs only (forward 4*Dh, backward 10*Dh per
 pair and query head) per second of the whole step, in TFLOP/s.
 
@@ -196,7 +197,7 @@ class HotPath:
         # the dQ accumulator is cleared on a side stream beside the forward (it needs
         # nothing from it), after the previous step's finalize has read it
         self.side = torch.cuda.Stream(device=dev)
-        self.ev_clear, self.ev_fin = torch.cuda.Event(), torch.cuda.Event()
+        self.ev_start, self.ev_clear, self.ev_fin = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
         self.launches_per_step = 5 + (1 if with_gather else 0)
 
     def _bufs(self):
@@ -207,7 +208,11 @@ class HotPath:
         b, s = self.b, self.s
         t = bufs or self._bufs()
         main = stream if stream is not None else torch.cuda.current_stream()
-        self.side.wait_event(self.ev_fin)  # the previous finalize has read the accumulator
+        # the side stream's clear starts only once this step has started on the main
+        # stream (so it is inside a timed step) and the previous step's dQ is out
+        self.ev_start.record(main)
+        self.side.wait_event(self.ev_start)
+        self.side.wait_event(self.ev_fin)
         b.sfa_bwd_clear(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, self.mode, self.ws, stream=self.side)
         self.ev_clear.record(self.side)
         if self.with_gather:
@@ -279,36 +284,47 @@ class HotPath:
         return h2d, d2h
 
 
-def time_loop(fn, steps, warmup, ws):
+class L2Flush:
+    """Writes a buffer of twice the L2 size, so the next timed region starts with none of
+    its inputs in L2."""
+
+    def __init__(self, dev):
+        self.nbytes = 2 * torch.cuda.get_device_properties(dev).L2_cache_size
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=dev)
+
+    def __call__(self):
+        self.buf.zero_()
+
+
+def timed_steps(step, iters: int, warmup: int, flush: L2Flush, ws: int = 1, nev: int = 4):
+    """Median device time (s) of `iters` calls of step(ev): each call bracketed by its own
+    CUDA events on the launching stream, the L2 flushed between calls outside the events,
+    `warmup` untimed calls first; ev holds `nev` events the step may record inside.
+    Returns (median step s, the per-step inner events)."""
     for _ in range(warmup):
-        fn()
+        step(None)
+        flush()
     torch.cuda.synchronize()
     barrier(ws)
     torch.cuda.synchronize()
-    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t0.record()
-    for _ in range(steps):
-        fn()
-    t1.record()
-    torch.cuda.synchronize()
-    barrier(ws)
-    return t0.elapsed_time(t1) / 1e3 / steps
-
-
-def measure_layer(s: AttnShape, mode: int, dev, iters=5, warmup=2, window: int = 0):
-    """fwd, bwd-main and fwd+bwd times of one layer (no gather), seconds."""
-    hp = HotPath(s, mode, dev, with_gather=False, seed=7, window=window)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(iters)]
-    for _ in range(warmup):
-        hp.step()
-    torch.cuda.synchronize()
-    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t0.record()
+    se = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(iters)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nev)] for _ in range(iters)]
     for i in range(iters):
-        hp.step(evs[i])
-    t1.record()
+        flush()
+        se[i][0].record()
+        step(evs[i])
+        se[i][1].record()
     torch.cuda.synchronize()
-    total = t0.elapsed_time(t1) / 1e3 / iters
+    barrier(ws)
+    return statistics.median(a.elapsed_time(b) for a, b in se) / 1e3, evs
+
+
+def measure_layer(s: AttnShape, mode: int, dev, iters=10, warmup=3, window: int = 0, flush=None):
+    """fwd, bwd-main and fwd+bwd times of one layer (no gather), seconds: medians over
+    `iters` steps with the L2 flushed between them."""
+    hp = HotPath(s, mode, dev, with_gather=False, seed=7, window=window)
+    flush = flush or L2Flush(dev)
+    total, evs = timed_steps(lambda ev: hp.step(ev), iters, warmup, flush)
     fwd = statistics.median(e[0].elapsed_time(e[1]) for e in evs) / 1e3
     bwd = statistics.median(e[2].elapsed_time(e[3]) for e in evs) / 1e3
     del hp
@@ -452,13 +468,14 @@ def final_pairs(L: int, n: int, mode: int, window: int = 0) -> int:
     return sum(min((t + 1) * n, window) for t in range(L))
 
 
-def measure_final_layer(dev, bf16_peak: float, iters: int = 5):
+def measure_final_layer(dev, bf16_peak: float, iters: int = 10, flush=None):
     """Final-stream-only layer (Sec. 3.1 KV-mirror layers: the L final-stream queries against
     all nL keys), L=4096, n=4, with Qwen3-8B-class heads (Hq=32, Hkv=8, Dh=128) and the 80B
     configuration's heads (Hq=24, Hkv=2, Dh=256, Table 6): fwd and bwd TFLOP/s over
-    visible pairs."""
+    visible pairs; medians over `iters` calls with the L2 flushed between them."""
     from paper_2607_08186_gb300 import binding
     B, L, n = 1, 4096, 4
+    flush = flush or L2Flush(dev)
     g = torch.Generator(device=dev)
     g.manual_seed(51)
 
@@ -475,8 +492,9 @@ def measure_final_layer(dev, bf16_peak: float, iters: int = 5):
         for mode in (WITHIN, CROSS):
             ws = torch.empty(binding.sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
                              device=dev)
-            tf = time_op(lambda k_: binding.sfa_fwd_final(q, k, v, o, lse, mode), 1, iters=iters)
-            tb = time_op(lambda k_: binding.sfa_bwd_final(q, k, v, o, lse, do, dq, dk, dv, mode, ws), 1, iters=iters)
+            tf, _ = timed_steps(lambda ev: binding.sfa_fwd_final(q, k, v, o, lse, mode), iters, 3, flush)
+            tb, _ = timed_steps(lambda ev: binding.sfa_bwd_final(q, k, v, o, lse, do, dq, dk, dv, mode, ws),
+                                iters, 3, flush)
             pairs = final_pairs(L, n, mode) * Hq * B
             res[MODE_NAME[mode]] = {"fwd_ms": tf * 1e3, "bwd_ms": tb * 1e3,
                                     "fwd_tflops": FWD_FLOP * Dh * pairs / tf / 1e12,
@@ -558,16 +576,17 @@ def source_hash(fname: str) -> str:
 
 def traffic_record(phase: str):
     """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
-    kernel behind `phase`, from profiles/traffic.md, if it was captured on the
-    current source of that kernel's file (else None)."""
+    kernel behind `phase`, from the ncu record profiles/traffic.json, if it was
+    captured on the current source of that kernel's file (else None)."""
     sym, fname = KERNEL_OF[phase]
-    path = os.path.join(ROOT, "profiles", "traffic.md")
+    path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
-    for ln in open(path):
-        cells = [c.strip() for c in ln.strip().strip("|").split("|")]
-        if len(cells) >= 4 and cells[0] == sym and cells[1] == fname:
-            return float(cells[3]) if cells[2] == source_hash(fname) else None
+    with open(path) as f:
+        rows = json.load(f).get("rows", [])
+    for r in rows:
+        if r.get("kernel") == sym and r.get("source") == fname:
+            return float(r["dram_bytes_per_launch"]) if r.get("sha16") == source_hash(fname) else None
     return None
 
 
@@ -679,7 +698,7 @@ def main():
             print(json.dumps(r), flush=True)
         return
     if args.final_only:
-        r = measure_final_layer(dev, pk["bf16"], iters=args.steps)
+        r = measure_final_layer(dev, pk["bf16"], iters=max(10, args.steps))
         if rank == 0:
             print(json.dumps(r), flush=True)
         return
@@ -708,34 +727,22 @@ def main():
     hp = HotPath(s, WITHIN, dev, with_gather=True, seed=1)
     flops_step = attn_flops(s, WITHIN, FWD_FLOP + BWD_FLOP)
 
-    # device-resident timed region
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
-    it = iter(range(10 ** 9))
+    # device-resident timed region: K steps, each bracketed by CUDA events on the
+    # launching stream, the L2 flushed (2 x L2 written) between steps outside the events;
+    # the step time is the median over the K steps
+    flush = L2Flush(dev)
     clocks = ClockSampler(local)
-
-    def timed():
-        i = next(it)
-        hp.step(evs[i - args.warmup] if i >= args.warmup else None)
-
     for _ in range(args.warmup):
-        timed()
+        hp.step()
+        flush()
     torch.cuda.synchronize()
-    barrier(ws)
     clocks.start()
     time.sleep(0.3)
-    torch.cuda.synchronize()
-    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t0.record()
-    for _ in range(args.steps):
-        timed()
-    t1.record()
-    torch.cuda.synchronize()
+    sec, evs = timed_steps(lambda ev: hp.step(ev), args.steps, 0, flush, ws)
     clk = clocks.stop()
-    barrier(ws)
-    sec = t0.elapsed_time(t1) / 1e3 / args.steps
     value, sec_max = job_throughput(flops_step, sec, ws)
-    fwd_s = statistics.mean(e[0].elapsed_time(e[1]) for e in evs) / 1e3
-    bwd_s = statistics.mean(e[2].elapsed_time(e[3]) for e in evs) / 1e3
+    fwd_s = statistics.median(e[0].elapsed_time(e[1]) for e in evs) / 1e3
+    bwd_s = statistics.median(e[2].elapsed_time(e[3]) for e in evs) / 1e3
     bwd_flops = attn_flops(s, WITHIN, BWD_FLOP)
     fwd_flops = attn_flops(s, WITHIN, FWD_FLOP)
     dom = "sfa_bwd_main" if bwd_s >= fwd_s else "sfa_fwd"
@@ -759,7 +766,11 @@ def main():
                                 f"Hq={s.Hq} Hkv={s.Hkv} Dh={s.Dh}, WITHIN mask, fwd+bwd, plus the "
                                 f"expansion gather of {s.n} tables {GATHER_V}x{GATHER_D}"),
                    "flops_per_step": flops_step, "flop_model": "fwd 4*Dh + bwd 10*Dh per visible pair per head",
-                   "l2": "inputs larger than L2 (Q 134 MB, dO 134 MB, K+V 67 MB, gather tables 5 GB)",
+                   "l2": (f"inputs larger than L2 (Q 134 MB, dO 134 MB, K+V 67 MB, gather tables 5 GB), and "
+                          f"the L2 flushed between steps ({flush.nbytes / 1e6:.0f} MB written, outside the "
+                          "steps' events)"),
+                   "timing": (f"median of {args.steps} steps, each bracketed by CUDA events on the launching "
+                              f"stream after {args.warmup} warm-up steps; max over ranks"),
                    "parallelism": f"replicas x{ws}"},
         "pct_of_peak": 100.0 * value / 1e12 / pk["bf16"],
         # the same step counted without the backward's QK^T recompute (bwd 8*Dh per pair)
@@ -778,7 +789,7 @@ def main():
     }
     if not args.no_extras and rank == 0 and ws == 1:
         extras = {}
-        r = measure_layer(s, CROSS, dev)
+        r = measure_layer(s, CROSS, dev, flush=flush)
         fl = attn_flops(s, CROSS, FWD_FLOP + BWD_FLOP)
         extras["cross_layer"] = {"workload": f"{WORKLOAD}_cross", "tflops": fl / r["step_s"] / 1e12,
                                  "fwd_tflops": attn_flops(s, CROSS, FWD_FLOP) / r["fwd_s"] / 1e12,
@@ -791,7 +802,7 @@ def main():
             # WITHIN_naive: WITHIN's mask per pair over the full causal tile schedule (no
             # stream-tile skipping), FLOPs counted over WITHIN's visible pairs
             for mode in (WITHIN, CROSS, WITHIN_NAIVE):
-                r = measure_layer(sn, mode, dev, iters=3, warmup=1)
+                r = measure_layer(sn, mode, dev, flush=flush)
                 fl = attn_flops(sn, mode, FWD_FLOP + BWD_FLOP)
                 row[MODE_NAME[mode]] = {"ms": r["step_s"] * 1e3, "tflops": fl / r["step_s"] / 1e12}
             row["skipping_speedup"] = row["WITHIN_naive"]["ms"] / row["WITHIN"]["ms"]
@@ -802,7 +813,7 @@ def main():
         extras["n_sweep"] = sweep
         loc = []
         for w in (1024, 4096):
-            r = measure_layer(s, LOCAL, dev, window=w)
+            r = measure_layer(s, LOCAL, dev, window=w, flush=flush)
             fl = attn_flops(s, LOCAL, FWD_FLOP + BWD_FLOP, w)
             loc.append({"window_positions": w, "ms": r["step_s"] * 1e3, "tflops": fl / r["step_s"] / 1e12,
                         "fwd_tflops": attn_flops(s, LOCAL, FWD_FLOP, w) / r["fwd_s"] / 1e12,
@@ -811,7 +822,7 @@ def main():
         # head dim 256 (80B-class heads: 24 query over 2 K/V heads): tcgen05 forward,
         # mma.sync backward
         s80 = AttnShape(1, 4096, 4, 24, 2, 256)
-        r = measure_layer(s80, WITHIN, dev, iters=3, warmup=1)
+        r = measure_layer(s80, WITHIN, dev, flush=flush)
         fl = attn_flops(s80, WITHIN, FWD_FLOP + BWD_FLOP)
         extras["head_dim_256_layer"] = {
             "workload": "B=1 L=4096 n=4 Hq=24 Hkv=2 Dh=256, WITHIN, fwd+bwd (tcgen05 forward, mma.sync backward)",
@@ -820,7 +831,7 @@ def main():
             "bwd_main_tflops": attn_flops(s80, WITHIN, BWD_FLOP) / r["bwd_main_s"] / 1e12}
         extras["expansion_backward"] = measure_expansion_backward(dev, pk["hbm"])
         extras["decode"] = measure_decode(dev, pk["hbm"], quick=True)
-        extras["final_stream_layer"] = measure_final_layer(dev, pk["bf16"])
+        extras["final_stream_layer"] = measure_final_layer(dev, pk["bf16"], flush=flush)
         extras["moe_stack"] = measure_moe_stack(dev, pk)
         out["extras"] = extras
         out["cpu_baseline"] = cpu_baseline()

@@ -277,9 +277,10 @@ hd_status_t sfa_kv_append(const void* k_new, const void* v_new, void* k_cache, v
  * long, present in every CUDA context that loads the library's module; the call
  * allocates and frees nothing.  Sizes whose sfa_bwd_workspace_bytes() exceeds that
  * limit return HD_ERR_SCRATCH_LIMIT before anything is enqueued (use sfa_bwd there).
- *   - Set-up: the first call on each device (current device at the time of the call)
- *     looks up the array's device address and keeps it; make that first call before
- *     any stream capture.  A failed look-up returns HD_ERR_CUDA.
+ *   - Set-up: every call looks up the array's device address in the calling thread's
+ *     current CUDA context (the address belongs to that context, so it is not cached);
+ *     the first call in a context also loads the library's module there, so make that
+ *     first call before any stream capture.  A failed look-up returns HD_ERR_CUDA.
  *   - Sharing: every call on a device uses the same array, which keeps the last call's
  *     contents; each call clears what it reads before reading it.  Calls that may run
  *     concurrently on one device (unordered streams, several host threads) race on

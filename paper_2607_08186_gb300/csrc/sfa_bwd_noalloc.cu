@@ -6,7 +6,7 @@
 // once it is serving, or plain C code with no device allocator at hand.  The call
 // allocates nothing: the array below is part of this module's static device image
 // (SFA_BWD_NOALLOC_MAX_BYTES of device memory in every CUDA context that loads the
-// module), and the entry point only looks up its address.
+// module), and the entry point only looks up its address in the current context.
 //
 // The array is shared by every call on a device and keeps the previous call's
 // contents.  Nothing stale is ever read: the prep pass of each call zeroes the fp32
@@ -14,8 +14,6 @@
 // main pass reads them.  Two calls that may run at the same time on one device
 // (different streams without an ordering event, or different host threads) use the
 // same array and race; the caller orders them.
-#include <mutex>
-
 #include "common.cuh"
 
 namespace {
@@ -25,32 +23,22 @@ static_assert(kScratchBytes % 256 == 0, "scratch size keeps the workspace split 
 
 static __device__ __align__(256) unsigned char g_sfa_bwd_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mu;
-void* g_scratch_addr[kMaxDevices];  // device address of the array on each device, looked up once
-
 bool aligned16(const void* p) { return p != nullptr && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Device address of the array on the current device.  The first call on a device
-// looks it up (which loads this module there if it is not loaded yet).
+// Device address of the array in the calling thread's current CUDA context.  The
+// address belongs to that context (a non-primary context on the same device, or the
+// primary context created again after cudaDeviceReset, holds the array elsewhere), so
+// it is looked up on every call instead of being cached per device; once the module
+// is loaded in the context the look-up is a table query.  The first call in a context
+// loads the module there.
 hd_status_t scratch_address(void** out) {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess) {
-    cudaGetLastError();
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_sfa_bwd_scratch);
+  if (e != cudaSuccess || p == nullptr) {
+    cudaGetLastError();  // leave no error behind for the caller's next check
     return HD_ERR_CUDA;
   }
-  if (dev < 0 || dev >= kMaxDevices) return HD_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lock(g_setup_mu);
-  if (g_scratch_addr[dev] == nullptr) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_sfa_bwd_scratch);
-    if (e != cudaSuccess || p == nullptr) {
-      cudaGetLastError();  // leave no error behind for the caller's next check
-      return HD_ERR_CUDA;
-    }
-    g_scratch_addr[dev] = p;
-  }
-  *out = g_scratch_addr[dev];
+  *out = p;
   return HD_OK;
 }
 

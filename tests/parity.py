@@ -99,3 +99,18 @@ def sample_rows(B, Hq, nL, count, seed, extra_p=()):
             rows.add((0, 0, p))
             rows.add((B - 1, Hq - 1, p))
     return np.array(sorted(rows), dtype=np.int64)
+
+
+def kv_sample_positions(nL, count, seed):
+    """Key positions for full-size dK / dV checks, spread over the whole sequence: the
+    first 128 positions (in a causal layer the keys that every later query sees, so
+    their gradients sum over the most query tiles and heads), a 128-position band in
+    the middle, and the last 384 positions (the shortest sums), plus both ends."""
+    g = torch.Generator().manual_seed(seed)
+    per = max(1, count // 3)
+    bands = [(0, min(128, nL)), (max(0, nL // 2 - 64), min(nL, nL // 2 + 64)), (max(0, nL - 384), nL)]
+    ps = {0, nL - 1}
+    for lo, hi in bands:
+        ps |= {int(x) for x in torch.randint(lo, hi, (per,), generator=g)}
+    return sorted(ps)
+

@@ -11,6 +11,8 @@ import torch
 import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
 
+from parity import kv_sample_positions
+
 pytestmark = pytest.mark.gpu
 
 WITHIN, CROSS, LOCAL = inputs.WITHIN, inputs.CROSS, inputs.LOCAL
@@ -104,7 +106,8 @@ def test_fwd_head_dim_64(mode):
 @pytest.mark.parametrize("mode", [WITHIN, CROSS])
 def test_full_size_sampled(mode):
     # Qwen3-8B-class heads, 4096 tokens, n = 4 (16384 key positions): every output row's
-    # forward statistics on sampled rows, dQ on sampled rows, dK / dV of the last 384 keys
+    # forward statistics on sampled rows, dQ on sampled rows, dK / dV of keys from the
+    # first 128 positions (the longest sums), a middle band and the last 384 positions
     B, L, n, Hq, Hkv, Dh = 1, 4096, 4, 32, 8, 128
     q, k, v, do = _inputs(B, L, n, Hq, Hkv, Dh, 11)
     got = _gpu(q, k, v, do, mode)
@@ -121,7 +124,7 @@ def test_full_size_sampled(mode):
     dq_r, _, _ = oracle.sfa_bwd_q_rows(qf, k, v, dof, n, mode, rows)
     dq_g = torch.stack([got["dq"][0, p // n, h] for (_, h, p) in rows])
     assert _rel(dq_g, dq_r) <= 1e-2
-    kv_rows = [(0, g, p) for g in (0, 7) for p in range(n * L - 384, n * L)]
+    kv_rows = [(0, g, p) for g in (0, 7) for p in kv_sample_positions(n * L, 48, 2)]
     dk_r, dv_r = oracle.sfa_bwd_kv_rows(qf, k, v, dof, n, mode, kv_rows)
     dk_g = torch.stack([got["dk"][0, p, g] for (_, g, p) in kv_rows])
     dv_g = torch.stack([got["dv"][0, p, g] for (_, g, p) in kv_rows])

@@ -14,7 +14,7 @@ from paper_2607_08186_gb300 import binding, build, inputs
 from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, WITHIN, WITHIN_NAIVE
 
 from parity import (assert_fwd_close, assert_grads_close, gpu_fwd, gpu_fwd_bwd, group_slices,
-                    max_abs, sample_rows, TOL_LSE, TOL_O)
+                    kv_sample_positions, max_abs, sample_rows, TOL_LSE, TOL_O)
 
 pytestmark = pytest.mark.gpu
 
@@ -176,11 +176,12 @@ def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
         assert max_abs(o_g, o_r) <= TOL_O
         assert max_abs(l_g, l_r) <= TOL_LSE
         assert_grads_close([("dq rows", dq[sel[:, 0], sel[:, 2], sel[:, 1]], dq_r)])
-    # dK / dV rows of one group: keys in the last 384 positions (complete sums
-    # over every query row and head of the group that sees them)
+    # dK / dV rows of one group, complete sums over every query row and head of the
+    # group that sees them: keys from the first 128 positions (the longest sums: every
+    # later query tile of the problem, all heads of the group), a band in the middle and
+    # the last 384 positions
     g = s.Hkv - 1
-    gen = torch.Generator().manual_seed(seed + 1)
-    ps = sorted({int(x) for x in torch.randint(s.nL - 384, s.nL, (n_kv,), generator=gen)} | {s.nL - 1})
+    ps = kv_sample_positions(s.nL, n_kv, seed + 1)
     kvrows = np.array([[0, 0, p] for p in ps], dtype=np.int64)
     qg, kg, vg, dog = group_slices(q, k, v, do, g, grp)
     dk_r, dv_r = oracle.sfa_bwd_kv_rows(qg, kg, vg, dog, s.n, mode, kvrows)
