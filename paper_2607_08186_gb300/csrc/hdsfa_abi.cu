@@ -40,6 +40,9 @@ cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v,
 cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                    void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
                                    const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
+cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* v, const void* dout, void* dk,
+                                      void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
+                                      const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
                                     float scale, cudaStream_t st);
 }  // namespace hdsfa
@@ -299,11 +302,14 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  // head dim 128 runs on the tcgen05 kernel; head dims 64 and 256 on the mma.sync kernel
-  // (at 256 as two CTAs per key tile, one per half of the dK / dV / dQ columns)
+  // head dims 128 and 256 run on the tcgen05 kernels (at 256 as two CTAs per key tile,
+  // one per half of the dK / dV / dQ columns); head dim 64 on the mma.sync kernel
   if (Dh == 128 && !use_mma_kernels())
     return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
                                                      scale, dev_status, stream));
+  if (Dh == 256 && !use_mma_kernels())
+    return cuda_status(hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
+                                                        scale, dev_status, stream));
   return cuda_status(hdsfa::launch_sfa_bwd_main_mma(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh,
                                                     scale, stream));
 }
@@ -436,7 +442,10 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
     if (Dh == 128 && !use_mma_kernels())
       e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status,
                                         stream);
-    else  // head dims 64 and 256 on the mma.sync kernel
+    else if (Dh == 256 && !use_mma_kernels())
+      e = hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status,
+                                           stream);
+    else  // head dim 64 on the mma.sync kernel
       e = hdsfa::launch_sfa_bwd_main_mma(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh, scale, stream);
   }
   if (e == cudaSuccess) e = hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, gq, Dh, scale, stream);
