@@ -558,11 +558,8 @@ def measure_decode(dev, hbm_peak: float, quick: bool = False):
 # ABI phase -> (kernel symbol, source file) of the implementation the library runs.
 KERNEL_OF = {
     "sfa_fwd": ("hdsfa::tcfwd::fwd_kernel<128, false>", "sfa_fwd_tc.cu"),
-    "sfa_bwd_main": ("hdsfa::tcbwd::bwd_kernel<false>", "sfa_bwd_tc.cu"),
+    "sfa_bwd_main": ("hdsfa::tcbwd::bwd_kernel<128, false>", "sfa_bwd_tc.cu"),
 }
-if os.environ.get("HDSFA_KERNELS") == "mma":
-    KERNEL_OF["sfa_fwd"] = ("hdsfa::sfa_fwd_mma_kernel<128>", "sfa_mma.cu")
-    KERNEL_OF["sfa_bwd_main"] = ("hdsfa::sfa_bwd_mma_kernel<128>", "sfa_mma.cu")
 
 
 def source_hash(fname: str) -> str:

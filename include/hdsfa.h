@@ -135,9 +135,8 @@ hd_status_t hd_select_final_stream_bwd(const void* dy, void* dx, int B, int L, i
  * q: bf16 [B][nL][Hq][Dh]; k, v: bf16 [B][nL][Hkv][Dh]; o: bf16 like q (written);
  * lse: float32 [B][Hq][nL] (written).  softmax_scale <= 0 selects 1/sqrt(Dh).
  * window is used only by SFA_LOCAL (must be >= 1 there).  Dh in {64, 128, 256}: the
- * forward runs on tcgen05 kernels at every head dim (256 is the paper's 80B
- * configuration, Table 6); the backward on tcgen05 at 128 and on warp-level mma.sync
- * kernels at 64 and 256.
+ * forward and the backward run on tcgen05 kernels at every head dim (256 is the
+ * paper's 80B configuration, Table 6).
  * Every position sees itself, so no softmax row is empty.
  */
 hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
@@ -213,8 +212,7 @@ hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int
  *   lse            : float32 [B][Hq][L], natural log (written by sfa_fwd_final)
  * dk, dv are fully overwritten (zero for keys no final-stream query sees).
  * workspace: >= sfa_bwd_final_workspace_bytes(...) bytes, 256-byte aligned.
- * Dh in {64, 128, 256}, on the same kernels as sfa_fwd / sfa_bwd (the forward on
- * tcgen05 kernels; the backward on tcgen05 at 128, on mma.sync at 64 and 256).
+ * Dh in {64, 128, 256}, on the same tcgen05 kernels as sfa_fwd / sfa_bwd.
  */
 hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
                           int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,

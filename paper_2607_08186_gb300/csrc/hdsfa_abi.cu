@@ -27,19 +27,13 @@ cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void*
                               const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_fwd_tc256(const void* q, const void* k, const void* v, void* o, float* lse,
                                  const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
-cudaError_t launch_sfa_fwd_mma(const void* q, const void* k, const void* v, void* o, float* lse,
-                               const SfaGeom& g, int Dh, float scale, cudaStream_t st);
 cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* lse, float* lse2_ws,
                                 float* delta_ws, float* dq_ws, const SfaGeom& g, int Dh,
                                 cudaStream_t st, bool zero = true);
 cudaError_t launch_sfa_bwd_clear(float* dq_ws, const SfaGeom& g, int Dh, cudaStream_t st);
-cudaError_t launch_sfa_bwd_main_mma(const void* q, const void* k, const void* v, const void* dout,
-                                    void* dk, void* dv, const float* lse2_ws, const float* delta_ws,
-                                    float* dq_ws, const SfaGeom& g, int Dh, float scale,
-                                    cudaStream_t st);
 cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                    void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
-                                   const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
+                                   const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                       void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
                                       const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
@@ -52,7 +46,6 @@ namespace {
 bool aligned16(const void* p) { return p != nullptr && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Validates sizes shared by sfa_fwd / sfa_bwd and builds the virtual-problem geometry.
-bool use_mma_kernels();
 
 hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, int window,
                       SfaGeom* g) {
@@ -62,8 +55,8 @@ hd_status_t make_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t m
     return HD_ERR_INVALID_ARG;
   if (mode == SFA_LOCAL && window <= 0) return HD_ERR_INVALID_ARG;
   if (Dh != 64 && Dh != 128 && Dh != 256) return HD_ERR_UNSUPPORTED;
-  // the naive schedule exists on the head-dim-128 tcgen05 kernels only
-  if (mode == SFA_WITHIN_NAIVE && (Dh != 128 || use_mma_kernels())) return HD_ERR_UNSUPPORTED;
+  // the naive schedule exists on the head-dim-128 kernels only
+  if (mode == SFA_WITHIN_NAIVE && Dh != 128) return HD_ERR_UNSUPPORTED;
   const long long nL = (long long)n * L;
   // Every row index, head product and tile count must fit the kernels' int math.
   if (nL > (1LL << 30) || (long long)B * nL * Hq > (1LL << 31) / 2) return HD_ERR_UNSUPPORTED;
@@ -116,17 +109,6 @@ hd_status_t make_final_geom(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mo
     g->kv_s0 = 0;
   }
   return HD_OK;
-}
-
-// HDSFA_KERNELS=mma selects the warp-level mma.sync kernels (the pre-tcgen05
-// baseline, kept for A/B timing); the default is the tcgen05 / TMA path.
-bool use_mma_kernels() {
-  static int v = -1;
-  if (v < 0) {
-    const char* e = getenv("HDSFA_KERNELS");
-    v = (e != nullptr && strcmp(e, "mma") == 0) ? 1 : 0;
-  }
-  return v == 1;
 }
 
 float resolve_scale(float s, int Dh) { return s > 0.f ? s : 1.0f / sqrtf((float)Dh); }
@@ -242,7 +224,6 @@ hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float*
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  if (use_mma_kernels()) return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
   // head dim 256: one query tile per CTA (its O takes half of TMEM)
   if (Dh == 256) return cuda_status(hdsfa::launch_sfa_fwd_tc256(q, k, v, o, lse, g, scale, dev_status, stream));
   return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
@@ -302,16 +283,13 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
   BwdWs ws;
   if ((st = split_ws(g, Dh, workspace, workspace_bytes, &ws)) != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  // head dims 128 and 256 run on the tcgen05 kernels (at 256 as two CTAs per key tile,
-  // one per half of the dK / dV / dQ columns); head dim 64 on the mma.sync kernel
-  if (Dh == 128 && !use_mma_kernels())
-    return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
-                                                     scale, dev_status, stream));
-  if (Dh == 256 && !use_mma_kernels())
+  // tcgen05 kernels at every head dim (at 256 as two CTAs per key tile, one per half
+  // of the dK / dV / dQ columns)
+  if (Dh == 256)
     return cuda_status(hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
                                                         scale, dev_status, stream));
-  return cuda_status(hdsfa::launch_sfa_bwd_main_mma(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh,
-                                                    scale, stream));
+  return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh,
+                                                   scale, dev_status, stream));
 }
 
 hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
@@ -405,7 +383,6 @@ hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, 
   hd_status_t st = make_final_geom(B, L, n, Hq, Hkv, Dh, mode, window, &g);
   if (st != HD_OK) return st;
   const float scale = resolve_scale(softmax_scale, Dh);
-  if (use_mma_kernels()) return cuda_status(hdsfa::launch_sfa_fwd_mma(q, k, v, o, lse, g, Dh, scale, stream));
   if (Dh == 256) return cuda_status(hdsfa::launch_sfa_fwd_tc256(q, k, v, o, lse, g, scale, dev_status, stream));
   return cuda_status(hdsfa::launch_sfa_fwd_tc(q, k, v, o, lse, g, Dh, scale, dev_status, stream));
 }
@@ -439,14 +416,12 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
     if (e == cudaSuccess) e = cudaMemsetAsync(dv, 0, bytes, stream);
   }
   if (e == cudaSuccess) {
-    if (Dh == 128 && !use_mma_kernels())
-      e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status,
-                                        stream);
-    else if (Dh == 256 && !use_mma_kernels())
+    if (Dh == 256)
       e = hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status,
                                            stream);
-    else  // head dim 64 on the mma.sync kernel
-      e = hdsfa::launch_sfa_bwd_main_mma(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh, scale, stream);
+    else
+      e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh, scale, dev_status,
+                                        stream);
   }
   if (e == cudaSuccess) e = hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, gq, Dh, scale, stream);
   return cuda_status(e);

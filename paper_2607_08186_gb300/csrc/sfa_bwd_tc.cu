@@ -1,5 +1,5 @@
 // Stream-Factorized Attention backward (main pass) on the sm_103a tensor cores,
-// head dim 128.
+// head dims 64 and 128 (template parameter DH).
 //
 // One CTA owns a 128-row key tile j of one virtual causal problem (SfaGeom) and
 // one K/V head; it loops over the group's query heads and over the 128-row query
@@ -59,14 +59,15 @@ namespace hdsfa {
 typedef __nv_bfloat16 bf16;
 
 namespace tcbwd {
-constexpr int BK = 128, BQ = 128, DH = 128, NTHREADS = 480;
+constexpr int BK = 128, BQ = 128, NTHREADS = 480;
 constexpr uint32_t COL_DV = 256, COL_DK = 384;
 HD_DEVINLINE uint32_t col_r(int r) { return 128u * r; }
 
+template <int DH>
 struct Smem {
-  bf16 k[BK * DH];        // 2 swizzle blocks of [128 key rows][64]
+  bf16 k[BK * DH];        // DH/64 swizzle blocks of [128 key rows][64]
   bf16 v[BK * DH];
-  bf16 q[2][BQ * DH];     // double-buffered query tile: 2 swizzle blocks of [128 rows][64]
+  bf16 q[2][BQ * DH];     // double-buffered query tile: DH/64 swizzle blocks of [128 rows][64]
   bf16 dO[BQ * DH];
   bf16 ds[BK * BQ];       // dS^T [128 key rows][128 queries]: 2 swizzle blocks of [128][64]
   float dqs[8][32 * 32];  // per dQ warp: [32 query rows][32 head-dim] fp32, 128-byte swizzle
@@ -74,14 +75,16 @@ struct Smem {
   float ndelta[2][BQ];    // -delta of the query tile in q[i], loaded with it
   uint64_t kv_full, q_full[2], q_empty[2], do_full, do_empty, s_full, dp_full, pa_part[4], pb_part[4], dq_full, s_init,
       dp_init, dk_done, dv_done, kv_done, drain;
+  uint64_t dq_read[DH == 64 ? 4 : 1];  // DH = 64: both dQ warps of a lane quadrant have read dQ(t)
   uint32_t tmem_base;
   int abort;
 };
 
 // The layout, 1024-byte aligned inside the dynamic shared memory, must fit the 227 KB
 // per-block limit; the kernel checks the actual alignment pad on entry.
-constexpr int kSmemBytes = 232448;
-static_assert(sizeof(Smem) <= kSmemBytes, "backward shared-memory layout exceeds 227 KB");
+template <int DH>
+constexpr int smem_bytes() { return (int)sizeof(Smem<DH>) + 1024 < 232448 ? (int)sizeof(Smem<DH>) + 1024 : 232448; }
+static_assert(sizeof(Smem<128>) <= 232448, "backward shared-memory layout exceeds 227 KB");
 
 struct Params {
   CUtensorMap tm_q, tm_do, tm_k, tm_v, tm_dq;
@@ -96,20 +99,23 @@ struct Params {
 
 
 // WIN: a windowed (LOCAL) problem, whose pre-fill masks only tiles that reach the
-// window edge; the other modes keep a separate instantiation.
-template <bool WIN>
+// window edge; the other modes keep a separate instantiation.  DH = 64: dQ, dK and
+// dV are 64 columns wide (N = 64 MMAs for dV, dK, dQ) and each dQ warp reads out 32
+// of them instead of 64; S^T, dP^T and the pre-fills are as at 128.
+template <int DH, bool WIN>
 __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant__ Params P) {
+  static_assert(DH == 64 || DH == 128, "head dim 64 or 128");
   extern __shared__ uint8_t smem_raw[];
   {
     uint32_t dyn;
     asm("mov.u32 %0, %%dynamic_smem_size;\n" : "=r"(dyn));
     const uintptr_t base = reinterpret_cast<uintptr_t>(smem_raw);
-    if (((base + 1023) & ~uintptr_t(1023)) - base + sizeof(Smem) > dyn) {  // uniform: nothing touched yet
+    if (((base + 1023) & ~uintptr_t(1023)) - base + sizeof(Smem<DH>) > dyn) {  // uniform: nothing touched yet
       if (threadIdx.x == 0) set_status(P.status, HD_DEVBIT_TIMEOUT);
       return;
     }
   }
-  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  Smem<DH>& sm = *reinterpret_cast<Smem<DH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // linear grid, key tile slowest: every CTA of key tile 0 (the most query tiles to
@@ -161,6 +167,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     mbar_init(&sm.dv_done, 1);
     mbar_init(&sm.kv_done, 1);
     mbar_init(&sm.drain, 2);
+    if (DH == 64)
+      for (int i = 0; i < 4; ++i) mbar_init(&sm.dq_read[i], 64);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -456,6 +464,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     // added into the fp32 accumulator by TMA reduce.
     const int dhalf = (warp - 6) >> 2;
     const int q4 = warp & 3;
+    constexpr int DQC = DH / 2;  // dQ columns read out and reduced by this warp
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     float* stage = sm.dqs[warp - 6];
     const float inv_c2 = 1.f / P.scale_log2;
@@ -560,10 +569,20 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         break;
       }
       tc_fence_after();
-      uint32_t v[64];
-      tmem_ld32(tl + col_r(p) + 64 * dhalf, v);
-      tmem_ld32(tl + col_r(p) + 64 * dhalf + 32, v + 32);
+      // this warp's DH/2 dQ columns [DQC*dhalf, +DQC)
+      uint32_t v[DQC];
+#pragma unroll
+      for (int r2 = 0; r2 < DQC / 32; ++r2) tmem_ld32(tl + col_r(p) + DQC * dhalf + 32 * r2, v + 32 * r2);
       tmem_ld_wait();
+      if constexpr (DH == 64) {
+        // the pre-fill below covers query columns [64*dhalf, +64) of R[p], which at DH = 64
+        // hold the other dQ warp's dQ columns: both warps of this quadrant read theirs first
+        mbar_arrive(&sm.dq_read[q4]);
+        if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_read[q4], t & 1, abort, P.status))) {
+          ok = false;
+          break;
+        }
+      }
       if (next) {
         // dQ(t) is out of R[p]: pre-fill it for dP'^T(t+1), 16 columns at a time
 #pragma unroll 1
@@ -583,7 +602,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         publish(&sm.dp_init);
       }
 #pragma unroll
-      for (int r2 = 0; r2 < 2; ++r2) {
+      for (int r2 = 0; r2 < DQC / 32; ++r2) {
         // the previous reduce from this warp's buffer must have read it
         if (lane == 0) bulk_wait_read0();
         __syncwarp();
@@ -595,7 +614,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         fence_async_smem();
         __syncwarp();
         if (lane == 0) {
-          tma_reduce_add_5d(&P.tm_dq, stage, 64 * dhalf + 32 * r2, h, s, q0 + q4 * 32, b);
+          tma_reduce_add_5d(&P.tm_dq, stage, DQC * dhalf + 32 * r2, h, s, q0 + q4 * 32, b);
           bulk_commit();
         }
       }
@@ -614,11 +633,25 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
 }
 }  // namespace tcbwd
 
+template <int DH>
+static cudaError_t bwd_tc_impl(tcbwd::Params& p, const SfaGeom& g, cudaStream_t st) {
+  using namespace tcbwd;
+  const int smem = smem_bytes<DH>();
+  auto kern = g.window > 0 ? bwd_kernel<DH, true> : bwd_kernel<DH, false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.q_ns * g.B);
+  kern<<<grid, NTHREADS, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+// Dh: 64 or 128.
 cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                    void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
-                                   const SfaGeom& g, float scale, int32_t* status, cudaStream_t st) {
+                                   const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st) {
   using namespace tcbwd;
   Params p;
+  const int DH = Dh;
   const SfaGeom gq = query_geom(g);
   if (!make_rows_tmap(&p.tm_q, q, gq, g.Hq, DH, BQ) || !make_rows_tmap(&p.tm_do, dout, gq, g.Hq, DH, BQ) ||
       !make_rows_tmap(&p.tm_k, k, g, g.Hkv, DH, BK) || !make_rows_tmap(&p.tm_v, v, g, g.Hkv, DH, BK) ||
@@ -632,13 +665,7 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   p.scale = scale;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.status = status;
-  const int smem = kSmemBytes;
-  auto kern = g.window > 0 ? bwd_kernel<true> : bwd_kernel<false>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
-  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.q_ns * g.B);
-  kern<<<grid, NTHREADS, smem, st>>>(p);
-  return cudaGetLastError();
+  return Dh == 64 ? bwd_tc_impl<64>(p, g, st) : bwd_tc_impl<128>(p, g, st);
 }
 
 }  // namespace hdsfa

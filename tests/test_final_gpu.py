@@ -83,8 +83,9 @@ def test_fwd_bwd_shapes(mode, w, B, L, n, Hq, Hkv):
 @pytest.mark.parametrize("B,L,n,Hq,Hkv,Dh", [(1, 70, 4, 24, 2, 256), (2, 40, 3, 4, 4, 256), (1, 90, 2, 4, 2, 64)])
 def test_head_dims_256_and_64_fwd_bwd(mode, w, B, L, n, Hq, Hkv, Dh):
     # head dim 256 (the 80B final-stream-only layers: 24 over 2 heads, Table 6) and head
-    # dim 64 run the final-stream geometry on their own kernels (head dim 256: the
-    # tcgen05 forward for that head dim and the mma.sync backward; 64: the mma.sync backward)
+    # dim 64 run the final-stream geometry on their own kernel instantiations (head dim
+    # 256: its own tcgen05 forward and the backward with two CTAs per key tile over the
+    # head-dim halves; 64: the head-dim-64 instantiation of the tcgen05 backward)
     q, k, v, do = _inputs(B, L, n, Hq, Hkv, Dh, L + Dh)
     got = _gpu(q, k, v, do, mode, w)
     o_r, lse_r = oracle.sfa_fwd_final(q, k, v, n, mode, window=w)

@@ -68,8 +68,8 @@ def test_wide_gqa_groups(mode, window):
 @pytest.mark.parametrize("mode,window", [(WITHIN, 0), (CROSS, 0), (LOCAL, 40)])
 def test_head_dim_256(mode, window):
     # head dim 256 (the paper's 80B configuration, 24 query over 2 K/V heads, Table 6):
-    # the forward on its own tcgen05 kernel, the backward on the mma.sync kernel as two
-    # CTAs per key tile over halves of the head dim
+    # the forward on its own tcgen05 kernel, the backward on the tcgen05 kernel with two
+    # CTAs per key tile over halves of the head dim and 64-row query tiles
     _full_case(AttnShape(1, 70, 4, 24, 2, 256), mode, seed=31, window=window)
     _full_case(AttnShape(2, 33, 2, 4, 4, 256), mode, seed=32, window=window)
 
