@@ -6,6 +6,7 @@
 
 #include "common.cuh"
 #include "decode_plan.cuh"
+#include "nvtx_range.h"
 
 namespace hdsfa {
 cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L,
@@ -154,6 +155,7 @@ extern "C" {
 
 hd_status_t hd_expand_embed(const void* tables, const int32_t* ids, void* out, int B, int L, int n,
                             int V, int D, int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_expand_embed");
   if (!aligned16(tables) || !aligned16(out) || ids == nullptr) return HD_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || n <= 0 || V <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
@@ -169,6 +171,7 @@ size_t hd_expand_embed_bwd_workspace_bytes(int B, int L) {
 
 hd_status_t hd_expand_embed_bwd_plan(const int32_t* ids, int B, int L, int V, void* workspace,
                                      size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_expand_embed_bwd_plan");
   if (ids == nullptr || (reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || V <= 0) return HD_ERR_INVALID_ARG;
   const size_t need = hd_expand_embed_bwd_workspace_bytes(B, L);
@@ -179,6 +182,7 @@ hd_status_t hd_expand_embed_bwd_plan(const int32_t* ids, int B, int L, int V, vo
 
 hd_status_t hd_expand_embed_bwd_apply(const void* dout, float* dtables, int B, int L, int n, int V, int D,
                                       const void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_expand_embed_bwd_apply");
   if (!aligned16(dout) || !aligned16(dtables)) return HD_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || n <= 0 || V <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
   const size_t need = hd_expand_embed_bwd_workspace_bytes(B, L);
@@ -190,6 +194,7 @@ hd_status_t hd_expand_embed_bwd_apply(const void* dout, float* dtables, int B, i
 hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dtables, int B, int L, int n,
                                 int V, int D, void* workspace, size_t workspace_bytes, int32_t* dev_status,
                                 cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_expand_embed_bwd");
   // every argument is checked before the plan is enqueued
   if (!aligned16(dout) || !aligned16(dtables) || ids == nullptr) return HD_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(ids) & 3u) != 0) return HD_ERR_INVALID_ARG;
@@ -203,6 +208,7 @@ hd_status_t hd_expand_embed_bwd(const void* dout, const int32_t* ids, float* dta
 }
 
 hd_status_t hd_select_final_stream(const void* x, void* y, int B, int L, int n, int D, cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_select_final_stream");
   if (!aligned16(x) || !aligned16(y)) return HD_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || n <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
   return cuda_status(hdsfa::launch_select_final(x, y, B, L, n, D, stream));
@@ -210,6 +216,7 @@ hd_status_t hd_select_final_stream(const void* x, void* y, int B, int L, int n, 
 
 hd_status_t hd_select_final_stream_bwd(const void* dy, void* dx, int B, int L, int n, int D,
                                        cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_select_final_stream_bwd");
   if (!aligned16(dy) || !aligned16(dx)) return HD_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || n <= 0 || D <= 0 || D % 8 != 0) return HD_ERR_INVALID_ARG;
   return cuda_status(hdsfa::launch_select_final_bwd(dy, dx, B, L, n, D, stream));
@@ -218,6 +225,7 @@ hd_status_t hd_select_final_stream_bwd(const void* dy, void* dx, int B, int L, i
 hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L,
                     int n, int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode,
                     int window, int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_fwd");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
     return HD_ERR_INVALID_ARG;
   SfaGeom g;
@@ -238,6 +246,7 @@ size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa
 hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int B, int L, int n, int Hq,
                          int Hkv, int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
                          cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_prep");
   if (!aligned16(o) || !aligned16(dout) || !aligned16(lse)) return HD_ERR_INVALID_ARG;
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
@@ -250,6 +259,7 @@ hd_status_t sfa_bwd_prep(const void* o, const void* dout, const float* lse, int 
 hd_status_t sfa_bwd_row_terms(const void* o, const void* dout, const float* lse, int B, int L, int n, int Hq,
                               int Hkv, int Dh, sfa_mode_t mode, void* workspace, size_t workspace_bytes,
                               cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_row_terms");
   if (!aligned16(o) || !aligned16(dout) || !aligned16(lse)) return HD_ERR_INVALID_ARG;
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
@@ -262,6 +272,7 @@ hd_status_t sfa_bwd_row_terms(const void* o, const void* dout, const float* lse,
 
 hd_status_t sfa_bwd_clear(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode, void* workspace,
                           size_t workspace_bytes, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_clear");
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
   if (st != HD_OK) return st;
@@ -274,6 +285,7 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
                          int B, int L, int n, int Hq, int Hkv, int Dh, float softmax_scale,
                          sfa_mode_t mode, int window, void* workspace, size_t workspace_bytes,
                          int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_main");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dout) || !aligned16(dk) ||
       !aligned16(dv))
     return HD_ERR_INVALID_ARG;
@@ -295,6 +307,7 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
 hd_status_t sfa_bwd_finalize(void* dq, int B, int L, int n, int Hq, int Hkv, int Dh,
                              float softmax_scale, sfa_mode_t mode, void* workspace,
                              size_t workspace_bytes, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_finalize");
   if (!aligned16(dq)) return HD_ERR_INVALID_ARG;
   SfaGeom g;
   hd_status_t st = make_geom(B, L, n, Hq, Hkv, Dh, mode, mode == SFA_LOCAL ? 1 : 0, &g);
@@ -310,6 +323,7 @@ hd_status_t sfa_bwd(const void* q, const void* k, const void* v, const void* o, 
                     int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
                     void* workspace, size_t workspace_bytes, int32_t* dev_status,
                     cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
       !aligned16(dout) || !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
     return HD_ERR_INVALID_ARG;
@@ -350,6 +364,7 @@ hd_status_t sfa_decode(const void* q, const void* k_cache, const void* v_cache, 
                        float* lse, int B, int max_tokens, int Lcap, int n, int Hq, int Hkv, int Dh,
                        float softmax_scale, sfa_mode_t mode, int window, void* workspace, size_t workspace_bytes,
                        int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_decode");
   if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(o)) return HD_ERR_INVALID_ARG;
   if (lens == nullptr || (reinterpret_cast<uintptr_t>(lens) & 3u) != 0) return HD_ERR_INVALID_ARG;
   if (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3u) != 0) return HD_ERR_INVALID_ARG;
@@ -364,6 +379,7 @@ hd_status_t sfa_decode(const void* q, const void* k_cache, const void* v_cache, 
 
 hd_status_t sfa_kv_append(const void* k_new, const void* v_new, void* k_cache, void* v_cache, const int32_t* lens,
                           int B, int Lcap, int n, int Hkv, int Dh, int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_kv_append");
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
     return HD_ERR_INVALID_ARG;
   if (lens == nullptr || (reinterpret_cast<uintptr_t>(lens) & 3u) != 0) return HD_ERR_INVALID_ARG;
@@ -377,6 +393,7 @@ hd_status_t sfa_kv_append(const void* k_new, const void* v_new, void* k_cache, v
 hd_status_t sfa_fwd_final(const void* q, const void* k, const void* v, void* o, float* lse, int B, int L, int n,
                           int Hq, int Hkv, int Dh, float softmax_scale, sfa_mode_t mode, int window,
                           int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_fwd_final");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
     return HD_ERR_INVALID_ARG;
   SfaGeom g;
@@ -397,6 +414,7 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
                           const void* dout, void* dq, void* dk, void* dv, int B, int L, int n, int Hq, int Hkv,
                           int Dh, float softmax_scale, sfa_mode_t mode, int window, void* workspace,
                           size_t workspace_bytes, int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_final");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
       !aligned16(dout) || !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
     return HD_ERR_INVALID_ARG;
@@ -428,6 +446,7 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
 }
 
 hd_status_t hd_selftest_bounded_wait(int32_t* dev_status, int32_t* dev_result, cudaStream_t stream) {
+  HD_NVTX_RANGE("hd_selftest_bounded_wait");
   if (dev_result == nullptr || (reinterpret_cast<uintptr_t>(dev_result) & 3u) != 0) return HD_ERR_INVALID_ARG;
   if (dev_status != nullptr && (reinterpret_cast<uintptr_t>(dev_status) & 3u) != 0) return HD_ERR_INVALID_ARG;
   return cuda_status(hdsfa::launch_bounded_wait_selftest(dev_status, dev_result, stream));

@@ -15,6 +15,7 @@
 // (different streams without an ordering event, or different host threads) use the
 // same array and race; the caller orders them.
 #include "common.cuh"
+#include "nvtx_range.h"
 
 namespace {
 
@@ -49,6 +50,7 @@ extern "C" hd_status_t sfa_bwd_noalloc(const void* q, const void* k, const void*
                                        int B, int L, int n, int Hq, int Hkv, int Dh,
                                        float softmax_scale, sfa_mode_t mode, int window,
                                        int32_t* dev_status, cudaStream_t stream) {
+  HD_NVTX_RANGE("sfa_bwd_noalloc");
   // argument errors answer as sfa_bwd does, before the array is looked at
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
       !aligned16(dout) || !aligned16(dq) || !aligned16(dk) || !aligned16(dv))

@@ -257,6 +257,9 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         for (int t = 0; ok && t < T; ++t) {
           const int p = t & 1;
           const uint64_t qM = p ? qM1 : qM0;
+          // dO(t) has landed (issuer Y waits for it too, but only before dP(t), which it
+          // may issue after phase A(t) has already released P^T(t) here)
+          if (!mbar_wait(&sm.do_full, t & 1, abort, P.status)) { ok = false; break; }
           for (int u = 0; u < 4; ++u) {
             if (!mbar_wait(&sm.pa_part[u], t & 1, abort, P.status)) { ok = false; break; }
             tc_fence_after();

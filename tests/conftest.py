@@ -20,3 +20,13 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+@pytest.fixture(autouse=True)
+def _output_guards(request):
+    """After every GPU test, the guard bytes around the outputs it allocated through
+    tests/guards.py must be intact."""
+    yield
+    if "gpu" in request.keywords:
+        import guards
+        guards.check_and_clear()

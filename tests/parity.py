@@ -11,6 +11,7 @@ from __future__ import annotations
 import numpy as np
 import torch
 
+import guards
 import oracle
 from paper_2607_08186_gb300 import binding
 
@@ -29,8 +30,8 @@ def check_status(st):
 def gpu_fwd(q, k, v, n, mode, scale=0.0, window=0, status=None):
     qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
     B, nL, Hq, Dh = q.shape
-    o = torch.empty_like(qd)
-    lse = torch.empty(B, Hq, nL, dtype=torch.float32, device="cuda")
+    o = guards.like(qd)
+    lse = guards.empty((B, Hq, nL), torch.float32)
     st = torch.zeros(1, dtype=torch.int32, device="cuda") if status is None else status
     binding.sfa_fwd(qd, kd, vd, o, lse, n, mode, scale or 0.0, window, dev_status=st)
     if status is None:
@@ -44,9 +45,9 @@ def gpu_fwd_bwd(q, k, v, do, n, mode, scale=0.0, window=0):
     dod = do.cuda()
     B, nL, Hq, Dh = q.shape
     Hkv = k.shape[2]
-    dq, dk, dv = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
+    dq, dk, dv = guards.like(qd), guards.like(kd), guards.like(vd)
     wsb = binding.sfa_bwd_workspace_bytes(B, nL // n, n, Hq, Hkv, Dh, mode)
-    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    ws = guards.empty((wsb,), torch.uint8, what="sfa_bwd workspace")
     binding.sfa_bwd(qd, kd, vd, o, lse, dod, dq, dk, dv, n, mode, ws, scale or 0.0, window, dev_status=st)
     check_status(st)
     return o.cpu(), lse.cpu(), dq.cpu(), dk.cpu(), dv.cpu()

@@ -6,6 +6,7 @@ accumulation, P rounded to bf16 for its MMA); the append is bit-exact."""
 import pytest
 import torch
 
+import guards
 import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
 
@@ -30,13 +31,13 @@ def _gpu_decode(q, kc, vc, lens, n, mode, window=0, max_tokens=None, status=None
     B, _, Hq, Dh = q.shape
     Lcap, Hkv = kc.shape[1] // n, kc.shape[2]
     T = Lcap if max_tokens is None else max_tokens
-    ws = torch.empty(binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode, window), dtype=torch.uint8,
-                     device="cuda")
+    ws = guards.empty((binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode, window),), torch.uint8,
+                      what="decode workspace")
     qd, kd, vd, ld = q.cuda(), kc.cuda(), vc.cuda(), lens.cuda()
     outs = []
     for _ in range(reps):
-        o = torch.full((B, n, Hq, Dh), 7.0, dtype=torch.bfloat16, device="cuda")
-        lse = torch.full((B, Hq, n), 7.0, dtype=torch.float32, device="cuda")
+        o = guards.empty((B, n, Hq, Dh), torch.bfloat16, 7.0)
+        lse = guards.empty((B, Hq, n), torch.float32, 7.0)
         binding.sfa_decode(qd, kd, vd, ld, o, n, mode, ws, max_tokens=T, lse=lse, window=window,
                            dev_status=status)
         torch.cuda.synchronize()
@@ -187,8 +188,8 @@ def test_serving_loop_in_a_cuda_graph(Hq, Hkv, Dh):
     # (head dim 256 with 24 over 2 heads: the tcgen05 decode kernel)
     B, n, Lcap = 2, 4, 64
     lens0 = [20, 33]
-    kc = torch.zeros(B, Lcap * n, Hkv, Dh, dtype=torch.bfloat16, device="cuda")
-    vc = torch.zeros_like(kc)
+    kc = guards.zeros((B, Lcap * n, Hkv, Dh), torch.bfloat16)
+    vc = guards.like(kc, 0)
     for b, t in enumerate(lens0):
         kc[b, :t * n] = inputs.normal_bf16((t * n, Hkv, Dh), 20 + b).cuda()
         vc[b, :t * n] = inputs.normal_bf16((t * n, Hkv, Dh), 30 + b).cuda()
@@ -197,10 +198,10 @@ def test_serving_loop_in_a_cuda_graph(Hq, Hkv, Dh):
     kn, vn = torch.zeros(B, n, Hkv, Dh, dtype=torch.bfloat16, device="cuda"), torch.zeros(B, n, Hkv, Dh,
                                                                                           dtype=torch.bfloat16,
                                                                                           device="cuda")
-    outs = {m: (torch.empty(B, n, Hq, Dh, dtype=torch.bfloat16, device="cuda"),
-                torch.empty(B, Hq, n, dtype=torch.float32, device="cuda")) for m in (WITHIN, CROSS)}
-    wss = {m: torch.empty(binding.sfa_decode_workspace_bytes(B, Lcap, n, Hq, Hkv, Dh, m), dtype=torch.uint8,
-                          device="cuda") for m in (WITHIN, CROSS)}
+    outs = {m: (guards.empty((B, n, Hq, Dh), torch.bfloat16), guards.empty((B, Hq, n), torch.float32))
+            for m in (WITHIN, CROSS)}
+    wss = {m: guards.empty((binding.sfa_decode_workspace_bytes(B, Lcap, n, Hq, Hkv, Dh, m),), torch.uint8)
+           for m in (WITHIN, CROSS)}
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
 
     def step():

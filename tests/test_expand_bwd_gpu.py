@@ -10,6 +10,7 @@ checked bitwise for repeatability."""
 import pytest
 import torch
 
+import guards
 import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
 
@@ -26,11 +27,13 @@ def _built():
 def _gpu_expand_bwd(dX, ids, n, V, dE0=None, status=None, reps=1):
     B, nL, D = dX.shape
     L = nL // n
-    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device="cuda")
+    ws = guards.empty((binding.hd_expand_embed_bwd_workspace_bytes(B, L),), torch.uint8, what="expand bwd ws")
     xd, idd = dX.cuda(), ids.cuda()
     outs = []
     for _ in range(reps):
-        dE = (torch.zeros(n, V, D, dtype=torch.float32) if dE0 is None else dE0.clone()).cuda()
+        dE = guards.zeros((n, V, D), torch.float32)
+        if dE0 is not None:
+            dE.copy_(dE0)
         binding.hd_expand_embed_bwd(xd, idd, dE, ws, dev_status=status)
         torch.cuda.synchronize()
         outs.append(dE.cpu())
@@ -108,7 +111,7 @@ def test_plan_once_apply_twice_on_another_stream():
     ids = inputs.token_ids(B, L, V, seed=15, zipf=1.0)
     dX1 = inputs.normal_bf16((B, n * L, D), seed=16)
     dX2 = inputs.normal_bf16((B, n * L, D), seed=17)
-    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device="cuda")
+    ws = guards.empty((binding.hd_expand_embed_bwd_workspace_bytes(B, L),), torch.uint8, what="expand bwd ws")
     side = torch.cuda.Stream()
     idd = ids.cuda()
     torch.cuda.synchronize()
@@ -117,11 +120,11 @@ def test_plan_once_apply_twice_on_another_stream():
         done = torch.cuda.Event()
         done.record(side)
     torch.cuda.current_stream().wait_event(done)
-    dE = torch.zeros(n, V, D, dtype=torch.float32, device="cuda")
+    dE = guards.zeros((n, V, D), torch.float32)
     binding.hd_expand_embed_bwd_apply(dX1.cuda(), dE, ws, L)
     torch.cuda.synchronize()
     _check_sum(dE.cpu(), dX1, ids, n, V)
-    dE2 = torch.zeros(n, V, D, dtype=torch.float32, device="cuda")
+    dE2 = guards.zeros((n, V, D), torch.float32)
     binding.hd_expand_embed_bwd_apply(dX2.cuda(), dE2, ws, L)
     torch.cuda.synchronize()
     _check_sum(dE2.cpu(), dX2, ids, n, V)
@@ -137,9 +140,9 @@ def test_apply_skips_what_the_plan_does_not_cover():
     B, L, n, V, D = 2, 700, 4, 300, 128
     ids = inputs.token_ids(B, L, V, seed=18, zipf=1.0)
     dX = inputs.normal_bf16((B, n * L, D), seed=19)
-    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device="cuda")
+    ws = guards.empty((binding.hd_expand_embed_bwd_workspace_bytes(B, L),), torch.uint8, what="expand bwd ws")
     binding.hd_expand_embed_bwd_plan(ids.cuda(), V, ws)
-    dE = torch.zeros(n, 150, D, dtype=torch.float32, device="cuda")
+    dE = guards.zeros((n, 150, D), torch.float32)
     binding.hd_expand_embed_bwd_apply(dX.cuda(), dE, ws, L)
     torch.cuda.synchronize()
     _check_sum(dE.cpu(), dX, ids, n, 150)
@@ -185,8 +188,8 @@ def test_full_size_sampled_ids():
     B, L, n, V, D = 1, 4096, 4, 151936, 4096
     dX = inputs.normal_bf16((B, n * L, D), seed=21)
     ids = inputs.token_ids(B, L, V, seed=21, zipf=1.0)
-    ws = torch.empty(binding.hd_expand_embed_bwd_workspace_bytes(B, L), dtype=torch.uint8, device="cuda")
-    dE = torch.zeros(n, V, D, dtype=torch.float32, device="cuda")
+    ws = guards.empty((binding.hd_expand_embed_bwd_workspace_bytes(B, L),), torch.uint8, what="expand bwd ws")
+    dE = guards.zeros((n, V, D), torch.float32)
     xd = dX.cuda()
     binding.hd_expand_embed_bwd(xd, ids.cuda(), dE, ws)
     torch.cuda.synchronize()
@@ -209,7 +212,7 @@ def test_full_size_sampled_ids():
 
 def _gpu_select(X, n):
     B, nL, D = X.shape
-    y = torch.full((B, nL // n, D), 7.0, dtype=torch.bfloat16, device="cuda")
+    y = guards.empty((B, nL // n, D), torch.bfloat16, 7.0)
     binding.hd_select_final_stream(X.cuda(), y, n)
     torch.cuda.synchronize()
     return y.cpu()
@@ -217,7 +220,7 @@ def _gpu_select(X, n):
 
 def _gpu_select_bwd(dY, n):
     B, L, D = dY.shape
-    dx = torch.full((B, n * L, D), 7.0, dtype=torch.bfloat16, device="cuda")
+    dx = guards.empty((B, n * L, D), torch.bfloat16, 7.0)
     binding.hd_select_final_stream_bwd(dY.cuda(), dx, n)
     torch.cuda.synchronize()
     return dx.cpu()

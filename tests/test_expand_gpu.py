@@ -3,6 +3,7 @@ import numpy as np
 import pytest
 import torch
 
+import guards
 import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
 
@@ -18,7 +19,7 @@ def _gpu_expand(tables, ids, status=None):
     n, V, D = tables.shape
     B, L = ids.shape
     td, idd = tables.cuda(), ids.cuda()
-    out = torch.full((B, n * L, D), 7.0, dtype=torch.bfloat16, device="cuda")
+    out = guards.empty((B, n * L, D), torch.bfloat16, 7.0)
     binding.hd_expand_embed(td, idd, out, dev_status=status)
     torch.cuda.synchronize()
     return out.cpu()

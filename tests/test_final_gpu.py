@@ -11,6 +11,7 @@ import torch
 import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
 
+import guards
 from parity import kv_sample_positions
 
 pytestmark = pytest.mark.gpu
@@ -36,15 +37,14 @@ def _gpu(q, k, v, do, mode, window=0, bwd=True):
     n, Hkv = k.shape[1] // L, k.shape[2]
     qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
-    o = torch.full((B, L, Hq, Dh), 7.0, dtype=torch.bfloat16, device="cuda")
-    lse = torch.full((B, Hq, L), 7.0, dtype=torch.float32, device="cuda")
+    o = guards.empty((B, L, Hq, Dh), torch.bfloat16, 7.0)
+    lse = guards.empty((B, Hq, L), torch.float32, 7.0)
     binding.sfa_fwd_final(qd, kd, vd, o, lse, mode, window=window, dev_status=st)
     out = {"o": o, "lse": lse}
     if bwd:
-        dq = torch.full_like(qd, 7.0)
-        dk, dv = torch.full_like(kd, 7.0), torch.full_like(vd, 7.0)
-        ws = torch.empty(binding.sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
-                         device="cuda")
+        dq = guards.like(qd, 7.0)
+        dk, dv = guards.like(kd, 7.0), guards.like(vd, 7.0)
+        ws = guards.empty((binding.sfa_bwd_final_workspace_bytes(B, L, n, Hq, Hkv, Dh, mode),), torch.uint8)
         binding.sfa_bwd_final(qd, kd, vd, o, lse, do.cuda(), dq, dk, dv, mode, ws, window=window, dev_status=st)
         out.update(dq=dq, dk=dk, dv=dv)
     torch.cuda.synchronize()

@@ -13,6 +13,7 @@ import oracle
 from paper_2607_08186_gb300 import binding, build, inputs
 from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, WITHIN, WITHIN_NAIVE
 
+import guards
 from parity import (assert_fwd_close, assert_grads_close, gpu_fwd, gpu_fwd_bwd, group_slices,
                     kv_sample_positions, max_abs, sample_rows, TOL_LSE, TOL_O)
 
@@ -126,11 +127,10 @@ def test_prep_halves_with_the_clear_on_a_side_stream(mode):
     s = AttnShape(1, 300, 4, 8, 2, 128)
     q, k, v, do = inputs.attn_inputs(s, seed=14)
     qd, kd, vd, dod = q.cuda(), k.cuda(), v.cuda(), do.cuda()
-    o = torch.empty_like(qd)
-    lse = torch.empty(s.B, s.Hq, s.nL, dtype=torch.float32, device="cuda")
+    o = guards.like(qd)
+    lse = guards.empty((s.B, s.Hq, s.nL), torch.float32)
     binding.sfa_fwd(qd, kd, vd, o, lse, s.n, mode)
-    ws = torch.full((binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),), 255,
-                    dtype=torch.uint8, device="cuda")
+    ws = guards.empty((binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),), torch.uint8, 255)
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(side):
@@ -139,11 +139,11 @@ def test_prep_halves_with_the_clear_on_a_side_stream(mode):
         cleared.record(side)
     binding.sfa_bwd_row_terms(o, dod, lse, s.n, mode, ws, s.Hkv)
     torch.cuda.current_stream().wait_event(cleared)
-    dq, dk, dv = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
+    dq, dk, dv = guards.like(qd), guards.like(kd), guards.like(vd)
     binding.sfa_bwd_main(qd, kd, vd, dod, dk, dv, s.n, mode, ws)
     binding.sfa_bwd_finalize(dq, s.n, mode, ws, s.Hkv)
-    dq1, dk1, dv1 = torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)
-    ws1 = torch.empty_like(ws)
+    dq1, dk1, dv1 = guards.like(qd), guards.like(kd), guards.like(vd)
+    ws1 = guards.like(ws)
     binding.sfa_bwd(qd, kd, vd, o, lse, dod, dq1, dk1, dv1, s.n, mode, ws1)
     torch.cuda.synchronize()
     dq_r, dk_r, dv_r = oracle.sfa_bwd(q, k, v, do, s.n, mode)
@@ -153,9 +153,15 @@ def test_prep_halves_with_the_clear_on_a_side_stream(mode):
 
 
 # ------------------------------------------------------------ full-size layers
-def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
+def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48, repeat=False):
     q, k, v, do = inputs.attn_inputs(s, seed=seed)
     o, lse, dq, dk, dv = gpu_fwd_bwd(q, k, v, do, s.n, mode)
+    if repeat:
+        # dK and dV are summed in a fixed order inside one CTA: a second run gives the
+        # same bits (an operand read before its load has landed would not)
+        _, _, _, dk2, dv2 = gpu_fwd_bwd(q, k, v, do, s.n, mode)
+        assert torch.equal(dk.view(torch.int16), dk2.view(torch.int16))
+        assert torch.equal(dv.view(torch.int16), dv2.view(torch.int16))
     if mode == WITHIN_NAIVE:  # checked against the WITHIN oracle
         mode = WITHIN
     grp = s.Hq // s.Hkv
@@ -191,19 +197,19 @@ def _sampled_parity(s: AttnShape, mode, seed, n_rows=192, n_kv=48):
 @pytest.mark.parametrize("mode", [WITHIN, CROSS, WITHIN_NAIVE])
 def test_qwen3_8b_class_layer(mode):
     # B=1, L=4096, n=4 (16384 positions), Hq=32, Hkv=8, Dh=128
-    _sampled_parity(inputs.SHAPES["qwen3_8b_n4"], mode, seed=1)
+    _sampled_parity(inputs.SHAPES["qwen3_8b_n4"], mode, seed=1, repeat=True)
 
 
 @pytest.mark.parametrize("mode", [WITHIN, CROSS])
 def test_large_moe_class_layer(mode):
     # B=1, L=8192, n=4 (32768 positions), Hq=64, Hkv=8, Dh=128
-    _sampled_parity(inputs.SHAPES["moe_large_n4"], mode, seed=21, n_rows=96, n_kv=24)
+    _sampled_parity(inputs.SHAPES["moe_large_n4"], mode, seed=21, n_rows=96, n_kv=24, repeat=True)
 
 
 @pytest.mark.parametrize("mode", [WITHIN, CROSS])
 def test_80b_class_layer(mode):
     # B=1, L=4096, n=4 (16384 positions), Hq=24, Hkv=2, Dh=256 (Table 6's 80B heads)
-    _sampled_parity(AttnShape(1, 4096, 4, 24, 2, 256), mode, seed=51, n_rows=64, n_kv=16)
+    _sampled_parity(AttnShape(1, 4096, 4, 24, 2, 256), mode, seed=51, n_rows=64, n_kv=16, repeat=True)
 
 
 @pytest.mark.parametrize("n", [1, 2, 8])

@@ -13,6 +13,7 @@ import torch
 from paper_2607_08186_gb300 import binding, build, inputs
 from paper_2607_08186_gb300.inputs import AttnShape, CROSS, LOCAL, WITHIN
 
+import guards
 from parity import assert_grads_close, check_status, gpu_fwd
 
 FAKE = 1 << 20  # 16-byte aligned non-null address; never dereferenced (validation fails first)
@@ -64,12 +65,10 @@ def test_calls_in_a_row_match_sfa_bwd(lib):
         st = torch.zeros(1, dtype=torch.int32, device="cuda")
         qd, kd, vd, o, lse = gpu_fwd(q, k, v, s.n, mode, 0.0, window, status=st)
         dod = do.cuda()
-        ref = [torch.empty_like(qd), torch.empty_like(kd), torch.empty_like(vd)]
-        ws = torch.empty(binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),
-                         dtype=torch.uint8, device="cuda")
+        ref = [guards.like(qd), guards.like(kd), guards.like(vd)]
+        ws = guards.empty((binding.sfa_bwd_workspace_bytes(s.B, s.L, s.n, s.Hq, s.Hkv, s.Dh, mode),), torch.uint8)
         binding.sfa_bwd(qd, kd, vd, o, lse, dod, *ref, s.n, mode, ws, 0.0, window, dev_status=st)
-        got = [torch.full_like(qd, float("nan")), torch.full_like(kd, float("nan")),
-               torch.full_like(vd, float("nan"))]
+        got = [guards.like(qd, float("nan")), guards.like(kd, float("nan")), guards.like(vd, float("nan"))]
         cases.append((s, mode, window, (qd, kd, vd, o, lse, dod), ref, got, st))
     # Two rounds of back-to-back calls on one stream.  The first noalloc call in this
     # context loads the module that holds the array (the one-time set-up), so the
