@@ -9,7 +9,12 @@
 // [B][L] tensors) against the same keys: query row r stands at key row
 // r*qstep + qoff, which sets its tile range and mask.
 //
-// Roles (320 threads; a CTA owns two 128-row query tiles, groups g = 0, 1):
+// A CTA owns two 128-row query tiles (groups g = 0, 1).  Where a K/V group has an
+// even number of query heads (GQA), they are the same rows of two of its heads, so
+// both see the same key tiles and finish together; otherwise rows m0 and m0 + 128 of
+// one head (the second tile then runs one key tile longer: measured as about 2 us of
+// a WITHIN CTA's 35 us, the first tile's softmax warps idle meanwhile).
+// Roles (320 threads):
 //   warp 0      TMA producer: both Q tiles once, then K/V tiles into a 2-stage ring;
 //               owns TMEM.
 //   warp 1      MMA issuer: the whole warp runs the issue loop, one elected lane
@@ -50,6 +55,7 @@ struct Params {
   SfaGeom g;
   float scale_log2;
   int32_t* status;
+  int head_pairs;  // 1: a CTA's two query tiles are the same rows of two heads of one K/V group
 };
 
 // Key row c visible from the query at key row rq (= r*qstep + qoff).
@@ -79,19 +85,31 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
   Smem<DH>& sm = *reinterpret_cast<Smem<DH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ncta = (G.Lq + NG * BM - 1) / (NG * BM);
+  // A CTA's two query tiles: with head_pairs the same 128 rows of heads 2x and 2x+1
+  // (one K/V group: both tiles see exactly the same key tiles and finish together),
+  // else rows m0 and m0 + 128 of one head (the second tile sees one more key tile).
+  const int hp = P.head_pairs;
+  const int rows_per_cta = hp ? BM : NG * BM;
+  const int ncta = (G.Lq + rows_per_cta - 1) / rows_per_cta;
+  const int nh = hp ? G.Hq / NG : G.Hq;  // head slots of the grid
   // linear grid, query-tile rank slowest: the last query tiles (the most key tiles to
   // visit) of every head, stream and batch launch first
-  const int per_rank = G.Hq * G.q_ns * G.B;
+  const int per_rank = nh * G.q_ns * G.B;
   const int mt = ncta - 1 - (int)blockIdx.x / per_rank;
   const int hsb = (int)blockIdx.x % per_rank;
-  const int m0 = mt * NG * BM;
-  const int b = hsb / (G.Hq * G.q_ns), h = (hsb / G.q_ns) % G.Hq, s = hsb % G.q_ns;
+  const int b = hsb / (nh * G.q_ns), hx = (hsb / G.q_ns) % nh, s = hsb % G.q_ns;
+  int qm[NG], hd[NG];  // first query row and head of each group's tile
+#pragma unroll
+  for (int g = 0; g < NG; ++g) {
+    qm[g] = hp ? mt * BM : mt * NG * BM + g * BM;
+    hd[g] = hp ? NG * hx + g : hx;
+  }
+  const int h = hd[0];
   const int sk = s + G.kv_s0;  // stream of the key problem
   const int kvh = h / (G.Hq / G.Hkv);
   int lo[NG], hi[NG];
 #pragma unroll
-  for (int g = 0; g < NG; ++g) tile_range(G, m0 + g * BM, lo[g], hi[g]);
+  for (int g = 0; g < NG; ++g) tile_range(G, qm[g], lo[g], hi[g]);
   const int n_lo = lo[0];
   int n_hi = hi[0];
 #pragma unroll
@@ -131,7 +149,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
       mbar_arrive_expect_tx(&sm.q_full, NG * BM * DH * 2);
       for (int g = 0; g < NG; ++g)
         for (int c = 0; c < DH / 64; ++c)
-          tma_load_5d(sm.q[g] + c * BM * 64, &P.tm_q, &sm.q_full, c * 64, h, s, m0 + g * BM, b);
+          tma_load_5d(sm.q[g] + c * BM * 64, &P.tm_q, &sm.q_full, c * 64, hd[g], s, qm[g], b);
       int issued = 0;
       for (int j = n_lo; j <= n_hi; ++j, ++issued) {
         const int it = j - n_lo, st = it % NST;
@@ -218,11 +236,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     const int g = (warp - 2) >> 2;
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
-    const int r = m0 + g * BM + row;
+    const int r = qm[g] + row;
+    const int hg = hd[g];
     const int rq = r * G.qstep + G.qoff;                      // its key row
-    const int rq0 = (m0 + g * BM) * G.qstep + G.qoff;         // key row of the tile's first query
+    const int rq0 = qm[g] * G.qstep + G.qoff;                 // key row of the tile's first query
     // key row of its last query (a key tile above rq1 - window is inside every row's window)
-    const int rq1 = (min(m0 + g * BM + BM, G.Lq) - 1) * G.qstep + G.qoff;
+    const int rq1 = (min(qm[g] + BM, G.Lq) - 1) * G.qstep + G.qoff;
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     const uint32_t tS = tl + g * 128, tO = tl + 256 + g * DH;
     const float c2 = P.scale_log2;
@@ -314,26 +333,44 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     if (ok && hi[g] >= lo[g] && __all_sync(0xffffffffu, mbar_wait(&sm.o_done[g], 0, abort, P.status))) {
       tc_fence_after();
       const float inv = 1.f / l_run;
-      bf16* orow = P.o + (((long long)b * G.q_nL + (long long)r * G.q_rs + s) * G.Hq + h) * DH;
+      // O rows leave through shared memory: each thread writes its row (normalised,
+      // bf16) into this warp's 32 rows of the group's Q buffer (no longer read: the last
+      // S MMA of the group completed before o_done), 16-byte units XOR-swizzled by the
+      // row; then every store instruction writes whole rows (DH*2 bytes each, 2 rows at
+      // DH = 128), instead of one 16-byte piece of 32 different rows.
+      constexpr int UPR = DH * 2 / 16;  // 16-byte units per row
+      uint8_t* stg = reinterpret_cast<uint8_t*>(sm.q[g]) + q4 * (32 * DH * 2);
 #pragma unroll
       for (int c = 0; c < DH / 32; ++c) {
         uint32_t o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_ld_wait();
-        if (r < G.Lq) {
 #pragma unroll
-          for (int e = 0; e < 32; e += 8) {
-            uint4 w;
-            w.x = cvt_bf16x2(__uint_as_float(o[e + 0]) * inv, __uint_as_float(o[e + 1]) * inv);
-            w.y = cvt_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
-            w.z = cvt_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv);
-            w.w = cvt_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv);
-            *reinterpret_cast<uint4*>(orow + c * 32 + e) = w;
-          }
+        for (int e = 0; e < 32; e += 8) {
+          uint4 w;
+          w.x = cvt_bf16x2(__uint_as_float(o[e + 0]) * inv, __uint_as_float(o[e + 1]) * inv);
+          w.y = cvt_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
+          w.z = cvt_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv);
+          w.w = cvt_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv);
+          const int u = c * 4 + e / 8;
+          *reinterpret_cast<uint4*>(stg + lane * (DH * 2) + ((u ^ (lane & 7)) << 4)) = w;
+        }
+      }
+      __syncwarp();
+      {
+        const long long rstride = (long long)G.q_rs * G.Hq * DH;  // elements between query rows
+        bf16* obase = P.o + (((long long)b * G.q_nL + s) * G.Hq + hg) * DH;
+        const int r0 = qm[g] + q4 * 32;  // this warp's first row
+#pragma unroll
+        for (int i = 0; i < 32 * UPR / 32; ++i) {
+          const int rr = (i * 32 + lane) / UPR, u = (i * 32 + lane) % UPR;  // row within the warp, unit
+          if (r0 + rr < G.Lq)
+            *reinterpret_cast<uint4*>(obase + (long long)(r0 + rr) * rstride + u * 8) =
+                *reinterpret_cast<const uint4*>(stg + rr * (DH * 2) + ((u ^ (rr & 7)) << 4));
         }
       }
       if (r < G.Lq)
-        P.lse[((long long)b * G.Hq + h) * G.q_nL + (long long)r * G.q_rs + s] = (m_run * c2 + log2f(l_run)) * kLn2;
+        P.lse[((long long)b * G.Hq + hg) * G.q_nL + (long long)r * G.q_rs + s] = (m_run * c2 + log2f(l_run)) * kLn2;
     }
   }
 
@@ -354,8 +391,9 @@ static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   cudaError_t e =
       cudaFuncSetAttribute(tcfwd::fwd_kernel<DH, NAIVE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const unsigned grid = (unsigned)((p.g.Lq + tcfwd::NG * tcfwd::BM - 1) / (tcfwd::NG * tcfwd::BM)) *
-                        (unsigned)(p.g.Hq * p.g.q_ns * p.g.B);
+  const int rows_per_cta = p.head_pairs ? tcfwd::BM : tcfwd::NG * tcfwd::BM;
+  const int nh = p.head_pairs ? p.g.Hq / tcfwd::NG : p.g.Hq;
+  const unsigned grid = (unsigned)((p.g.Lq + rows_per_cta - 1) / rows_per_cta) * (unsigned)(nh * p.g.q_ns * p.g.B);
   tcfwd::fwd_kernel<DH, NAIVE><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
   return cudaGetLastError();
 }
@@ -372,6 +410,7 @@ cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void*
   p.g = g;
   p.scale_log2 = scale * tcfwd::kLog2e;
   p.status = status;
+  p.head_pairs = (g.Hq / g.Hkv) % tcfwd::NG == 0;
   if (Dh == 64) return tc_fwd_impl<64, false>(p, st);
   return g.smod > 1 ? tc_fwd_impl<128, true>(p, st) : tc_fwd_impl<128, false>(p, st);
 }
