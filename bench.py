@@ -816,13 +816,13 @@ def main():
                         "fwd_tflops": attn_flops(s, LOCAL, FWD_FLOP, w) / r["fwd_s"] / 1e12,
                         "bwd_main_tflops": attn_flops(s, LOCAL, BWD_FLOP, w) / r["bwd_main_s"] / 1e12})
         extras["local_layer"] = {"workload": f"{WORKLOAD}_local", "windows": loc}
-        # head dim 256 (80B-class heads: 24 query over 2 K/V heads): tcgen05 forward,
-        # mma.sync backward
+        # head dim 256 (80B-class heads: 24 query over 2 K/V heads): the head-dim-256
+        # tcgen05 forward and backward kernels
         s80 = AttnShape(1, 4096, 4, 24, 2, 256)
         r = measure_layer(s80, WITHIN, dev, flush=flush)
         fl = attn_flops(s80, WITHIN, FWD_FLOP + BWD_FLOP)
         extras["head_dim_256_layer"] = {
-            "workload": "B=1 L=4096 n=4 Hq=24 Hkv=2 Dh=256, WITHIN, fwd+bwd (tcgen05 forward, mma.sync backward)",
+            "workload": "B=1 L=4096 n=4 Hq=24 Hkv=2 Dh=256, WITHIN, fwd+bwd (head-dim-256 tcgen05 kernels)",
             "ms": r["step_s"] * 1e3, "tflops": fl / r["step_s"] / 1e12,
             "fwd_tflops": attn_flops(s80, WITHIN, FWD_FLOP) / r["fwd_s"] / 1e12,
             "bwd_main_tflops": attn_flops(s80, WITHIN, BWD_FLOP) / r["bwd_main_s"] / 1e12}
