@@ -349,6 +349,32 @@ def time_op(fn, sets: int, iters=21, warmup=3):
     return a.elapsed_time(b) / 1e3 / iters
 
 
+def time_graph(fn, sets: int, reps: int = 7, warmup: int = 3):
+    """Device time (s) per call of fn(k) when `reps` rounds over the `sets` buffer sets
+    are captured once as a CUDA graph and replayed: what a serving loop that replays
+    its step graph pays, without the host's launch cost per call."""
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(stream):
+        for k in range(warmup):
+            fn(k % sets)
+    torch.cuda.current_stream().wait_stream(stream)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for k in range(reps * sets):
+            fn(k % sets)
+    graph.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    del graph
+    return a.elapsed_time(b) / 1e3 / (reps * sets)
+
+
 def measure_expansion_backward(dev, hbm_peak: float, V: int = GATHER_V):
     """Expansion backward (adjoint of Eq. 1) and final-stream selection (Eq. 2) with
     its adjoint at the step's shapes: L=4096 tokens, n=4, D=4096, V=151936.
@@ -511,8 +537,12 @@ def measure_decode(dev, hbm_peak: float, quick: bool = False):
     """Decoding step (Sec. 3.2), n=4: the new token's 4 positions against a context of T
     tokens (4T cached positions) for batch B, WITHIN and CROSS layers, with Qwen3-8B-class
     heads (Hq=32, Hkv=8, Dh=128) and, unless quick, the 80B configuration's heads (Hq=24,
-    Hkv=2, Dh=256) and the 617B configuration's (Hq=96, Hkv=8, Dh=128) of Table 6.  Algorithmic bytes: the visible cached K and V rows (B*T*n*Hkv*Dh*2 bytes
-    each) plus q and o; rotating cache sets keep every call out of L2."""
+    Hkv=2, Dh=256) and the 617B configuration's (Hq=96, Hkv=8, Dh=128) of Table 6.
+    Algorithmic bytes: the visible cached K and V rows (B*T*n*Hkv*Dh*2 bytes each) plus
+    q and o; rotating cache sets keep every call out of L2.  `us` is the device time per
+    step of the calls replayed from a CUDA graph (how a serving loop runs the step);
+    `us_eager` the same calls launched one by one from Python, where at batch 1 the
+    host's launch cost per call is about the kernels' time."""
     from paper_2607_08186_gb300 import binding
     n = 4
     heads = {"qwen3_8b": (32, 8, 128, [(1, 8192), (4, 8192), (16, 8192), (1, 32768), (16, 32768)]),
@@ -541,11 +571,13 @@ def measure_decode(dev, hbm_peak: float, quick: bool = False):
             for mode in (WITHIN, CROSS):
                 ws = torch.empty(binding.sfa_decode_workspace_bytes(B, T, n, Hq, Hkv, Dh, mode), dtype=torch.uint8,
                                  device=dev)
-                t = time_op(lambda k: binding.sfa_decode(sets[k][0], sets[k][1], sets[k][2], lens, o, n, mode, ws,
-                                                         max_tokens=T, lse=lse), S)
+                call = (lambda k: binding.sfa_decode(sets[k][0], sets[k][1], sets[k][2], lens, o, n, mode, ws,
+                                                     max_tokens=T, lse=lse))
+                t = time_graph(call, S)
+                te = time_op(call, S)
                 nbytes = cache_bytes + 2 * B * n * Hq * Dh * 2
                 row[MODE_NAME[mode]] = {"us": t * 1e6, "gbs": nbytes / t / 1e9,
-                                        "frac_hbm": nbytes / t / 1e9 / hbm_peak}
+                                        "frac_hbm": nbytes / t / 1e9 / hbm_peak, "us_eager": te * 1e6}
             out.append(row)
             del sets, o, lse
             torch.cuda.empty_cache()
