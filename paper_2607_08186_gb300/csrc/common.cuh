@@ -55,6 +55,25 @@ __host__ __device__ inline SfaGeom query_geom(const SfaGeom& g) {
 constexpr int kRowTermAlign = 128;
 __host__ __device__ inline int row_terms_pitch(int Lv) { return (Lv + kRowTermAlign - 1) / kRowTermAlign * kRowTermAlign; }
 
+// Head chunks of the head-dim-256 backward.  Its grid is two CTAs per 128-row key tile
+// and (b, K/V head, stream); when that is fewer than two CTAs per SM (short or
+// final-stream problems with few K/V heads), each CTA takes only a chunk of the group's
+// query heads, and the chunks' dK / dV partial sums meet in an fp32 workspace
+// [2][B][q_ns][Lv][Hkv][256] (dV, then dK already scaled) that a finalize pass converts.
+constexpr int kSmCount = 152;
+__host__ __device__ inline int bwd256_head_chunks(const SfaGeom& g) {
+  const long long ctas = (long long)((g.Lv + 127) / 128) * 2 * g.Hkv * g.q_ns * g.B;
+  const int grp = g.Hq / g.Hkv;
+  if (ctas >= 2 * kSmCount || grp < 2) return 1;
+  long long want = (2 * kSmCount + ctas - 1) / ctas;
+  const int hs = (int)(want < grp ? want : grp);
+  const int per = (grp + hs - 1) / hs;
+  return (grp + per - 1) / per;
+}
+__host__ __device__ inline size_t bwd256_dkv_elems(const SfaGeom& g) {  // of one of dV, dK
+  return bwd256_head_chunks(g) > 1 ? (size_t)g.B * g.q_ns * g.Lv * g.Hkv * 256 : 0;
+}
+
 HD_DEVINLINE uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

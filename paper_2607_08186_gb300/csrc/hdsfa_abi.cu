@@ -37,7 +37,8 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
                                    const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
 cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                       void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
-                                      const SfaGeom& g, float scale, int32_t* status, cudaStream_t st);
+                                      float* dkv_ws, const SfaGeom& g, float scale, int32_t* status,
+                                      cudaStream_t st);
 cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
                                     float scale, cudaStream_t st);
 }  // namespace hdsfa
@@ -117,11 +118,14 @@ float resolve_scale(float s, int Dh) { return s > 0.f ? s : 1.0f / sqrtf((float)
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then -lse*log2(e) and
-// -delta, each fp32 [B][Hq][ns][Lvp] (stream-major rows, Lvp = row_terms_pitch(Lv)).
+// -delta, each fp32 [B][Hq][ns][Lvp] (stream-major rows, Lvp = row_terms_pitch(Lv)),
+// then at head dim 256 on small grids the fp32 dV / dK partial sums of the head chunks
+// (bwd256_dkv_elems each).
 struct BwdWs {
   float* dq;
   float* lse2;
   float* delta;
+  float* dkv;
 };
 
 // Sizes follow the query side (query_geom): the accumulator and row terms are per query row.
@@ -129,7 +133,8 @@ size_t ws_bytes(const SfaGeom& gk, int Dh) {
   const SfaGeom g = query_geom(gk);
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
   const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)row_terms_pitch(g.Lv);
-  return align256(rows * Dh * sizeof(float)) + 2 * align256(trows * sizeof(float));
+  const size_t dkv = Dh == 256 ? 2 * bwd256_dkv_elems(gk) * sizeof(float) : 0;
+  return align256(rows * Dh * sizeof(float)) + 2 * align256(trows * sizeof(float)) + align256(dkv);
 }
 
 hd_status_t split_ws(const SfaGeom& gk, int Dh, void* ws, size_t bytes, BwdWs* out) {
@@ -144,6 +149,8 @@ hd_status_t split_ws(const SfaGeom& gk, int Dh, void* ws, size_t bytes, BwdWs* o
   out->lse2 = reinterpret_cast<float*>(p);
   p += align256(trows * sizeof(float));
   out->delta = reinterpret_cast<float*>(p);
+  p += align256(trows * sizeof(float));
+  out->dkv = Dh == 256 && bwd256_dkv_elems(gk) > 0 ? reinterpret_cast<float*>(p) : nullptr;
   return HD_OK;
 }
 
@@ -298,7 +305,7 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
   // tcgen05 kernels at every head dim (at 256 as two CTAs per key tile, one per half
   // of the dK / dV / dQ columns)
   if (Dh == 256)
-    return cuda_status(hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g,
+    return cuda_status(hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, ws.dkv, g,
                                                         scale, dev_status, stream));
   return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh,
                                                    scale, dev_status, stream));
@@ -435,7 +442,7 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
   }
   if (e == cudaSuccess) {
     if (Dh == 256)
-      e = hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, scale, dev_status,
+      e = hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, ws.dkv, g, scale, dev_status,
                                            stream);
     else
       e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh, scale, dev_status,

@@ -27,6 +27,10 @@
 //   head-dim column.)  dQ_c^T(t) lands in RS(p) once P^T(t) is consumed, leaves TMEM
 //   through the dQ warps, staged in shared memory over the dS^T buffer (free once
 //   dQ_c^T has read it) and added into the fp32 accumulator by TMA tensor reduce-add.
+// Small grids (fewer than two CTAs per SM: short or final-stream problems with two K/V
+// heads) also split the group's query heads into chunks, one CTA each; the chunks' dK /
+// dV partial sums are added into an fp32 workspace (red.global.add) and converted by
+// dkv_finalize_kernel (bwd256_head_chunks in common.cuh).
 // Roles (512 threads, at most 128 registers each): warp 0 TMA producer (+ TMEM owner);
 // three MMA issuers on different warps, each waiting only for its own operands:
 // warp 1 (one lane) dV_c and dK_c per 16-query quarter, warp 14 (whole warp, an
@@ -75,6 +79,8 @@ struct Params {
   const float* delta;  // [B][Hq][ns][Lvp]
   bf16* dk;
   bf16* dv;
+  float* dkv;   // head chunks > 1: fp32 partial sums [2][B][q_ns][Lv][Hkv][DH] (dV, dK)
+  int hchunks;  // query-head chunks per K/V head (bwd256_head_chunks)
   SfaGeom g;
   float scale, scale_log2;
   int32_t* status;
@@ -98,16 +104,20 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
   const SfaGeom& G = P.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // linear grid, key tile slowest (the tiles with the most query tiles first); the two
-  // head-dim halves of a key tile are neighbours
-  const int per_tile = 2 * G.Hkv * G.q_ns * G.B;
+  // head-dim halves of a key tile are neighbours, then its head chunks
+  const int HC = P.hchunks;
+  const int per_tile = 2 * HC * G.Hkv * G.q_ns * G.B;
   const int j = (int)blockIdx.x / per_tile;
   const int rem = (int)blockIdx.x % per_tile;
-  const int c = rem & 1, hsb = rem >> 1;
+  const int c = rem & 1, hc = (rem >> 1) % HC, hsb = (rem >> 1) / HC;
   const int o = c ^ 1;
   const int n0 = j * BK;
   const int b = hsb / (G.Hkv * G.q_ns), kvh = (hsb / G.q_ns) % G.Hkv, s = hsb % G.q_ns;
   const int sk = s + G.kv_s0;  // stream of the key problem
-  const int grp = G.Hq / G.Hkv;
+  // this CTA's query heads: chunk hc of the group's grp heads
+  const int grp_all = G.Hq / G.Hkv, hper = (grp_all + HC - 1) / HC;
+  const int grp = min(hper, grp_all - hc * hper);  // heads of this chunk (>= 1)
+  const int h_base = kvh * grp_all + hc * hper;
   // query rows that can see a key of the tile: key row r*qstep + qoff >= n0, and under
   // a window r*qstep + qoff < n0 + BK - 1 + window
   const int i_lo = (n0 <= G.qoff ? 0 : (n0 - G.qoff + G.qstep - 1) / G.qstep) / BQ;
@@ -117,6 +127,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
   const int T = grp * nq;
   const int Lqp = row_terms_pitch(G.Lq);
   if (nq <= 0) {  // no query sees this key tile: its half of the dK and dV rows is zero
+    if (HC > 1) return;  // the workspace rows stay zero; the finalize pass writes them
     for (int i = threadIdx.x; i < BK * (DHH / 8); i += NTHREADS) {
       const int kr = n0 + i / (DHH / 8), cc = i % (DHH / 8);
       if (kr >= G.Lv) continue;
@@ -179,7 +190,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
       // the query tile t: its other half once S^T(t-1)'s first k-steps are done, its own
       // half into qc[t&1] once dK_c(t-2) is done; dO(t) once dV_c(t-1) and dP(t-1) are
       for (int t = 0; t < T; ++t) {
-        const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
+        const int h = h_base + t / nq, q0 = (i_lo + t % nq) * BQ;
         const int qb = t & 1;
         if (t >= 1 && !mbar_wait(&sm.qo_empty, (t - 1) & 1, abort, P.status)) break;
         if (t >= 2 && !mbar_wait(&sm.qc_empty[qb], ((t - 2) >> 1) & 1, abort, P.status)) break;
@@ -387,10 +398,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
         }
       }
     }
-    // epilogue: this key row's half of dV, then of dK (scaled)
+    // epilogue: this key row's half of dV, then of dK (scaled); with head chunks, added
+    // into the fp32 workspace instead (red.global.add, 16 bytes at a time)
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
       tc_fence_after();
       const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + sk) * G.Hkv + kvh) * DH + c * DHH;
+      const size_t half = (size_t)G.B * G.q_ns * G.Lv * G.Hkv * DH;
+      const long long wrow = ((((long long)b * G.q_ns + s) * G.Lv + kr) * G.Hkv + kvh) * DH + c * DHH;
 #pragma unroll 1
       for (int cc = 0; cc < 2 * DHH / 32; ++cc) {
         const int which = cc >= DHH / 32;
@@ -400,7 +414,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
         uint32_t ov[32];
         tmem_ld32(tl + col, ov);
         tmem_ld_wait();
-        if (kr < G.Lv) {
+        if (HC > 1) {
+          if (kr < G.Lv) {
+            float* wdst = P.dkv + which * half + wrow + (cc % (DHH / 32)) * 32;
+#pragma unroll
+            for (int e = 0; e < 32; e += 4)
+              red_add_v4(wdst + e, __uint_as_float(ov[e]) * mul, __uint_as_float(ov[e + 1]) * mul,
+                         __uint_as_float(ov[e + 2]) * mul, __uint_as_float(ov[e + 3]) * mul);
+          }
+        } else if (kr < G.Lv) {
 #pragma unroll
           for (int e = 0; e < 32; e += 8) {
             uint4 w;
@@ -492,7 +514,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
     }
     for (int t = 0; ok && t < T; ++t) {
       const int p = t & 1, ph = (t >> 1) & 1;
-      const int h = kvh * grp + t / nq, q0 = tile_q0(t);
+      const int h = h_base + t / nq, q0 = tile_q0(t);
       const bool refill = t + 2 < T;
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.dq_full[p], ph, abort, P.status))) {
         ok = false;
@@ -557,11 +579,39 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
     tmem_dealloc(tmem, 512);
   }
 }
+// Head chunks: dv / dk rows (bf16) from the fp32 partial sums, 8 columns per thread.
+__global__ void __launch_bounds__(256) dkv_finalize_kernel(const float* __restrict__ dkv, bf16* __restrict__ dk,
+                                                           bf16* __restrict__ dv, SfaGeom g) {
+  const long long n8 = (long long)g.B * g.q_ns * g.Lv * g.Hkv * (DH / 8);
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n8) return;
+  const int c8 = (int)(i % (DH / 8));
+  long long r = i / (DH / 8);
+  const int kvh = (int)(r % g.Hkv);
+  r /= g.Hkv;
+  const int kr = (int)(r % g.Lv);
+  r /= g.Lv;
+  const int s = (int)(r % g.q_ns), b = (int)(r / g.q_ns);
+  const long long orow = (((long long)b * g.nL + (long long)kr * g.rs + s + g.kv_s0) * g.Hkv + kvh) * DH + c8 * 8;
+  const size_t half = (size_t)n8 * 8;
+#pragma unroll
+  for (int which = 0; which < 2; ++which) {
+    const float4* src = reinterpret_cast<const float4*>(dkv + which * half + i * 8);
+    const float4 x = src[0], y = src[1];
+    uint4 w;
+    w.x = cvt_bf16x2(x.x, x.y);
+    w.y = cvt_bf16x2(x.z, x.w);
+    w.z = cvt_bf16x2(y.x, y.y);
+    w.w = cvt_bf16x2(y.z, y.w);
+    *reinterpret_cast<uint4*>((which ? dk : dv) + orow) = w;
+  }
+}
 }  // namespace tcbwd256
 
 cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                       void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
-                                      const SfaGeom& g, float scale, int32_t* status, cudaStream_t st) {
+                                      float* dkv_ws, const SfaGeom& g, float scale, int32_t* status,
+                                      cudaStream_t st) {
   using namespace tcbwd256;
   Params p;
   const SfaGeom gq = query_geom(g);
@@ -573,16 +623,28 @@ cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* 
   p.delta = delta_ws;
   p.dk = (bf16*)dk;
   p.dv = (bf16*)dv;
+  p.hchunks = bwd256_head_chunks(g);
+  p.dkv = dkv_ws;
   p.g = g;
   p.scale = scale;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.status = status;
+  const size_t nkv = bwd256_dkv_elems(g);
+  if (p.hchunks > 1) {
+    if (dkv_ws == nullptr) return cudaErrorInvalidValue;
+    cudaError_t e = cudaMemsetAsync(dkv_ws, 0, 2 * nkv * sizeof(float), st);
+    if (e != cudaSuccess) return e;
+  }
   const int smem = kSmemBytes;
   auto kern = g.window > 0 ? bwd256_kernel<true> : bwd256_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(2 * g.Hkv * g.q_ns * g.B);
+  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(2 * p.hchunks * g.Hkv * g.q_ns * g.B);
   kern<<<grid, NTHREADS, smem, st>>>(p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || p.hchunks == 1) return e;
+  const long long n8 = (long long)nkv / 8;
+  dkv_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dkv_ws, (bf16*)dk, (bf16*)dv, g);
   return cudaGetLastError();
 }
 
