@@ -144,7 +144,9 @@ hd_status_t sfa_fwd(const void* q, const void* k, const void* v, void* o, float*
                     int window, int32_t* dev_status, cudaStream_t stream);
 
 /* Bytes of device workspace sfa_bwd needs for these sizes and mode (fp32 dQ
- * accumulator [B][nL][Hq][Dh] plus two fp32 row terms of about B*Hq*nL each).
+ * accumulator [B][nL][Hq][Dh] plus two fp32 row terms of about B*Hq*nL each; when the
+ * backward's grid would leave SMs idle, also fp32 dK and dV partial sums [B][nL][Hkv][Dh]
+ * for each of the query-head chunks it then splits the work into).
  * Returns 0 for invalid sizes. */
 size_t sfa_bwd_workspace_bytes(int B, int L, int n, int Hq, int Hkv, int Dh, sfa_mode_t mode);
 

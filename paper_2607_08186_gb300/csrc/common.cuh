@@ -55,23 +55,28 @@ __host__ __device__ inline SfaGeom query_geom(const SfaGeom& g) {
 constexpr int kRowTermAlign = 128;
 __host__ __device__ inline int row_terms_pitch(int Lv) { return (Lv + kRowTermAlign - 1) / kRowTermAlign * kRowTermAlign; }
 
-// Head chunks of the head-dim-256 backward.  Its grid is two CTAs per 128-row key tile
-// and (b, K/V head, stream); when that is fewer than two CTAs per SM (short or
+// Head chunks of the tensor-core backward.  Its grid is one CTA (two at head dim 256)
+// per 128-row key tile and (b, K/V head, stream); when that leaves SMs idle (short or
 // final-stream problems with few K/V heads), each CTA takes only a chunk of the group's
-// query heads, and the chunks' dK / dV partial sums meet in an fp32 workspace
-// [2][B][q_ns][Lv][Hkv][256] (dV, then dK already scaled) that a finalize pass converts.
+// query heads, for about two CTAs per SM.  (With one to two CTAs per SM, as in the n = 1
+// and the final-stream intra-stream layers with 8 K/V heads, the partial sums' extra
+// traffic cost more than the better balance gained: 3 % slower.)  Chunk hc writes its dK / dV partial sums (fp32,
+// dK already scaled) to its own slice of a workspace [chunks][2][B][q_ns][Lv][Hkv][Dh]
+// (dV, then dK), and a finalize pass adds the slices in chunk order: the same result,
+// bit for bit, on every run.
 constexpr int kSmCount = 152;
-__host__ __device__ inline int bwd256_head_chunks(const SfaGeom& g) {
-  const long long ctas = (long long)((g.Lv + 127) / 128) * 2 * g.Hkv * g.q_ns * g.B;
+__host__ __device__ inline int bwd_head_chunks(const SfaGeom& g, int Dh) {
+  const long long ctas = (long long)((g.Lv + 127) / 128) * (Dh == 256 ? 2 : 1) * g.Hkv * g.q_ns * g.B;
   const int grp = g.Hq / g.Hkv;
-  if (ctas >= 2 * kSmCount || grp < 2) return 1;
+  if (ctas >= kSmCount || grp < 2) return 1;
   long long want = (2 * kSmCount + ctas - 1) / ctas;
   const int hs = (int)(want < grp ? want : grp);
   const int per = (grp + hs - 1) / hs;
   return (grp + per - 1) / per;
 }
-__host__ __device__ inline size_t bwd256_dkv_elems(const SfaGeom& g) {  // of one of dV, dK
-  return bwd256_head_chunks(g) > 1 ? (size_t)g.B * g.q_ns * g.Lv * g.Hkv * 256 : 0;
+// Elements of one slice half (dV or dK of one chunk); 0 without chunks.
+__host__ __device__ inline size_t bwd_dkv_slice(const SfaGeom& g, int Dh) {
+  return bwd_head_chunks(g, Dh) > 1 ? (size_t)g.B * g.q_ns * g.Lv * g.Hkv * Dh : 0;
 }
 
 HD_DEVINLINE uint32_t smem_u32(const void* p) {

@@ -34,7 +34,8 @@ cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* ls
 cudaError_t launch_sfa_bwd_clear(float* dq_ws, const SfaGeom& g, int Dh, cudaStream_t st);
 cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                    void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
-                                   const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st);
+                                   float* dkv_ws, const SfaGeom& g, int Dh, float scale, int32_t* status,
+                                   cudaStream_t st);
 cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                       void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
                                       float* dkv_ws, const SfaGeom& g, float scale, int32_t* status,
@@ -119,8 +120,8 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Workspace layout: fp32 dQ accumulator [B][nL][Hq][Dh], then -lse*log2(e) and
 // -delta, each fp32 [B][Hq][ns][Lvp] (stream-major rows, Lvp = row_terms_pitch(Lv)),
-// then at head dim 256 on small grids the fp32 dV / dK partial sums of the head chunks
-// (bwd256_dkv_elems each).
+// then on small grids the fp32 dV / dK partial sums of the head chunks, one slice per
+// chunk (bwd_dkv_slice elements each).
 struct BwdWs {
   float* dq;
   float* lse2;
@@ -133,7 +134,7 @@ size_t ws_bytes(const SfaGeom& gk, int Dh) {
   const SfaGeom g = query_geom(gk);
   const size_t rows = (size_t)g.B * g.nL * g.Hq;
   const size_t trows = (size_t)g.B * g.Hq * g.ns * (size_t)row_terms_pitch(g.Lv);
-  const size_t dkv = Dh == 256 ? 2 * bwd256_dkv_elems(gk) * sizeof(float) : 0;
+  const size_t dkv = (size_t)bwd_head_chunks(gk, Dh) * 2 * bwd_dkv_slice(gk, Dh) * sizeof(float);
   return align256(rows * Dh * sizeof(float)) + 2 * align256(trows * sizeof(float)) + align256(dkv);
 }
 
@@ -150,7 +151,7 @@ hd_status_t split_ws(const SfaGeom& gk, int Dh, void* ws, size_t bytes, BwdWs* o
   p += align256(trows * sizeof(float));
   out->delta = reinterpret_cast<float*>(p);
   p += align256(trows * sizeof(float));
-  out->dkv = Dh == 256 && bwd256_dkv_elems(gk) > 0 ? reinterpret_cast<float*>(p) : nullptr;
+  out->dkv = bwd_dkv_slice(gk, Dh) > 0 ? reinterpret_cast<float*>(p) : nullptr;
   return HD_OK;
 }
 
@@ -307,7 +308,7 @@ hd_status_t sfa_bwd_main(const void* q, const void* k, const void* v, const void
   if (Dh == 256)
     return cuda_status(hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, ws.dkv, g,
                                                         scale, dev_status, stream));
-  return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh,
+  return cuda_status(hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, ws.dkv, g, Dh,
                                                    scale, dev_status, stream));
 }
 
@@ -445,7 +446,7 @@ hd_status_t sfa_bwd_final(const void* q, const void* k, const void* v, const voi
       e = hdsfa::launch_sfa_bwd_main_tc256(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, ws.dkv, g, scale, dev_status,
                                            stream);
     else
-      e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, g, Dh, scale, dev_status,
+      e = hdsfa::launch_sfa_bwd_main_tc(q, k, v, dout, dk, dv, ws.lse2, ws.delta, ws.dq, ws.dkv, g, Dh, scale, dev_status,
                                         stream);
   }
   if (e == cudaSuccess) e = hdsfa::launch_sfa_bwd_finalize(dq, ws.dq, gq, Dh, scale, stream);

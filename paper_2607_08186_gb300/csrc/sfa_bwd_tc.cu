@@ -40,6 +40,10 @@
 // one thread execute in order), so it overlaps the dQ(t) read-out; dP(t+1) lands in
 // R[p] only after that read-out.
 //
+// Small grids (fewer CTAs than SMs) also split the group's query heads into chunks, one
+// CTA each; each chunk writes its fp32
+// dK / dV partial sums to a workspace slice of its own, which dkv_finalize_kernel adds
+// in chunk order (bwd_head_chunks in common.cuh).
 // Roles (480 threads, 128 registers each): warp 0 TMA producer (+ TMEM owner);
 // warp 1 MMA issuer X (dV, dK per query quarter; one lane); warp 14 MMA issuer Y
 // (dQ, S, dP; the whole warp runs its loop, one elected lane issues, 0.7 % faster than
@@ -92,6 +96,8 @@ struct Params {
   const float* delta;  // [B][Hq][ns][Lvp]
   bf16* dk;
   bf16* dv;
+  float* dkv;   // head chunks > 1: fp32 partial sums [chunks][2][B][q_ns][Lv][Hkv][DH] (dV, dK)
+  int hchunks;  // query-head chunks per K/V head (bwd_head_chunks)
   SfaGeom g;
   float scale, scale_log2;
   int32_t* status;
@@ -120,13 +126,19 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // linear grid, key tile slowest: every CTA of key tile 0 (the most query tiles to
   // visit) launches before any of tile 1, and so on, over all heads, streams and batches
-  const int per_tile = G.Hkv * G.q_ns * G.B;
+  // (and head chunks, neighbours)
+  const int HC = P.hchunks;
+  const int per_tile = HC * G.Hkv * G.q_ns * G.B;
   const int j = (int)blockIdx.x / per_tile;
-  const int hsb = (int)blockIdx.x % per_tile;
+  const int rem = (int)blockIdx.x % per_tile;
+  const int hc = rem % HC, hsb = rem / HC;
   const int n0 = j * BK;
   const int b = hsb / (G.Hkv * G.q_ns), kvh = (hsb / G.q_ns) % G.Hkv, s = hsb % G.q_ns;
   const int sk = s + G.kv_s0;  // stream of the key problem
-  const int grp = G.Hq / G.Hkv;
+  // this CTA's query heads: chunk hc of the group's heads
+  const int grp_all = G.Hq / G.Hkv, hper = (grp_all + HC - 1) / HC;
+  const int grp = min(hper, grp_all - hc * hper);  // heads of this chunk (>= 1)
+  const int h_base = kvh * grp_all + hc * hper;
   // query rows that can see a key of the tile: key row r*qstep + qoff >= n0, and under
   // a window r*qstep + qoff < n0 + BK - 1 + window
   const int i_lo = (n0 <= G.qoff ? 0 : (n0 - G.qoff + G.qstep - 1) / G.qstep) / BQ;
@@ -136,6 +148,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
   const int T = grp * nq;
   const int Lqp = row_terms_pitch(G.Lq);
   if (nq <= 0) {  // no query sees this key tile: its dK and dV rows are zero
+    if (HC > 1) {  // this chunk's slice rows are zero
+      const size_t half = (size_t)G.B * G.q_ns * G.Lv * G.Hkv * DH;
+      for (int i = threadIdx.x; i < BK * (DH / 4); i += NTHREADS) {
+        const int kr = n0 + i / (DH / 4), c4 = i % (DH / 4);
+        if (kr >= G.Lv) continue;
+        const long long wrow = ((((long long)b * G.q_ns + s) * G.Lv + kr) * G.Hkv + kvh) * DH + c4 * 4;
+        *reinterpret_cast<float4*>(P.dkv + (2 * hc) * half + wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
+        *reinterpret_cast<float4*>(P.dkv + (2 * hc + 1) * half + wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      return;
+    }
     for (int i = threadIdx.x; i < BK * (DH / 8); i += NTHREADS) {
       const int kr = n0 + i / (DH / 8), c = i % (DH / 8);
       if (kr >= G.Lv) continue;
@@ -197,7 +220,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
       int nq_issued = 0, ndo_issued = 0;
       // query tiles (with their row terms) run up to two ahead (double buffer); dO one ahead
       for (int t = 0; t < T; ++t) {
-        const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
+        const int h = h_base + t / nq, q0 = (i_lo + t % nq) * BQ;
         const int qb = t & 1;
         if (t >= 2 && !mbar_wait(&sm.q_empty[qb], ((t - 2) >> 1) & 1, abort, P.status)) break;
         mbar_arrive_expect_tx(&sm.q_full[qb], BQ * DH * 2 + 2 * BQ * 4);
@@ -430,10 +453,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         }
       }
     }
-    // epilogue: this key row of dV, then of dK (scaled)
+    // epilogue: this key row of dV, then of dK (scaled); with head chunks, into this
+    // chunk's fp32 workspace slice instead
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
       tc_fence_after();
       const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + sk) * G.Hkv + kvh) * DH;
+      const size_t half = (size_t)G.B * G.q_ns * G.Lv * G.Hkv * DH;
+      const long long wrow = ((((long long)b * G.q_ns + s) * G.Lv + kr) * G.Hkv + kvh) * DH;
 #pragma unroll 1
       for (int c = 0; c < 2 * DH / 32; ++c) {
         const int which = c >= DH / 32;
@@ -443,7 +469,16 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
         uint32_t o[32];
         tmem_ld32(tl + col, o);
         tmem_ld_wait();
-        if (kr < G.Lv) {
+        if (HC > 1) {
+          if (kr < G.Lv) {
+            float* wdst = P.dkv + (2 * hc + which) * half + wrow + (c % (DH / 32)) * 32;
+#pragma unroll
+            for (int e = 0; e < 32; e += 4)
+              *reinterpret_cast<float4*>(wdst + e) =
+                  make_float4(__uint_as_float(o[e]) * mul, __uint_as_float(o[e + 1]) * mul,
+                              __uint_as_float(o[e + 2]) * mul, __uint_as_float(o[e + 3]) * mul);
+          }
+        } else if (kr < G.Lv) {
 #pragma unroll
           for (int e = 0; e < 32; e += 8) {
             uint4 w;
@@ -549,7 +584,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     }
     for (int t = 0; ok && t < T; ++t) {
       const int p = t & 1;
-      const int h = kvh * grp + t / nq, q0 = (i_lo + t % nq) * BQ;
+      const int h = h_base + t / nq, q0 = (i_lo + t % nq) * BQ;
       const bool next = t + 1 < T;
       if (next) {
         // R[p^1] for S'^T(t+1): row terms of tile t+1 loaded; dK(t) has read dS^T(t) there
@@ -634,24 +669,65 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     tmem_dealloc(tmem, 512);
   }
 }
+// Head chunks: dv / dk rows (bf16) from the chunks' fp32 partial sums, added in chunk
+// order, 8 columns per thread.
+template <int DH>
+__global__ void __launch_bounds__(256) dkv_finalize_kernel(const float* __restrict__ dkv, bf16* __restrict__ dk,
+                                                           bf16* __restrict__ dv, SfaGeom g, int chunks) {
+  const long long n8 = (long long)g.B * g.q_ns * g.Lv * g.Hkv * (DH / 8);
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n8) return;
+  const int c8 = (int)(i % (DH / 8));
+  long long r = i / (DH / 8);
+  const int kvh = (int)(r % g.Hkv);
+  r /= g.Hkv;
+  const int kr = (int)(r % g.Lv);
+  r /= g.Lv;
+  const int s = (int)(r % g.q_ns), b = (int)(r / g.q_ns);
+  const long long orow = (((long long)b * g.nL + (long long)kr * g.rs + s + g.kv_s0) * g.Hkv + kvh) * DH + c8 * 8;
+  const size_t half = (size_t)n8 * 8;
+#pragma unroll
+  for (int which = 0; which < 2; ++which) {
+    float4 x = make_float4(0.f, 0.f, 0.f, 0.f), y = x;
+    for (int hc = 0; hc < chunks; ++hc) {
+      const float4* src = reinterpret_cast<const float4*>(dkv + (2 * hc + which) * half + i * 8);
+      const float4 a = src[0], e = src[1];
+      x.x += a.x; x.y += a.y; x.z += a.z; x.w += a.w;
+      y.x += e.x; y.y += e.y; y.z += e.z; y.w += e.w;
+    }
+    uint4 w;
+    w.x = cvt_bf16x2(x.x, x.y);
+    w.y = cvt_bf16x2(x.z, x.w);
+    w.z = cvt_bf16x2(y.x, y.y);
+    w.w = cvt_bf16x2(y.z, y.w);
+    *reinterpret_cast<uint4*>((which ? dk : dv) + orow) = w;
+  }
+}
 }  // namespace tcbwd
 
 template <int DH>
 static cudaError_t bwd_tc_impl(tcbwd::Params& p, const SfaGeom& g, cudaStream_t st) {
   using namespace tcbwd;
+  const size_t nkv = bwd_dkv_slice(g, DH);
+  if (p.hchunks > 1 && p.dkv == nullptr) return cudaErrorInvalidValue;
   const int smem = smem_bytes<DH>();
   auto kern = g.window > 0 ? bwd_kernel<DH, true> : bwd_kernel<DH, false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(g.Hkv * g.q_ns * g.B);
+  const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(p.hchunks * g.Hkv * g.q_ns * g.B);
   kern<<<grid, NTHREADS, smem, st>>>(p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || p.hchunks == 1) return e;
+  const long long n8 = (long long)nkv / 8;
+  dkv_finalize_kernel<DH><<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(p.dkv, p.dk, p.dv, g, p.hchunks);
   return cudaGetLastError();
 }
 
 // Dh: 64 or 128.
 cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, const void* dout, void* dk,
                                    void* dv, const float* lse2_ws, const float* delta_ws, float* dq_ws,
-                                   const SfaGeom& g, int Dh, float scale, int32_t* status, cudaStream_t st) {
+                                   float* dkv_ws, const SfaGeom& g, int Dh, float scale, int32_t* status,
+                                   cudaStream_t st) {
   using namespace tcbwd;
   Params p;
   const int DH = Dh;
@@ -664,6 +740,8 @@ cudaError_t launch_sfa_bwd_main_tc(const void* q, const void* k, const void* v, 
   p.delta = delta_ws;
   p.dk = (bf16*)dk;
   p.dv = (bf16*)dv;
+  p.hchunks = bwd_head_chunks(g, Dh);
+  p.dkv = dkv_ws;
   p.g = g;
   p.scale = scale;
   p.scale_log2 = scale * 1.4426950408889634f;

@@ -27,10 +27,10 @@
 //   head-dim column.)  dQ_c^T(t) lands in RS(p) once P^T(t) is consumed, leaves TMEM
 //   through the dQ warps, staged in shared memory over the dS^T buffer (free once
 //   dQ_c^T has read it) and added into the fp32 accumulator by TMA tensor reduce-add.
-// Small grids (fewer than two CTAs per SM: short or final-stream problems with two K/V
-// heads) also split the group's query heads into chunks, one CTA each; the chunks' dK /
-// dV partial sums are added into an fp32 workspace (red.global.add) and converted by
-// dkv_finalize_kernel (bwd256_head_chunks in common.cuh).
+// Small grids (fewer CTAs than SMs: short or final-stream problems with two K/V heads)
+// also split the group's query heads into chunks, one CTA each; each chunk
+// writes its fp32 dK / dV partial sums to a workspace slice of its own, which
+// dkv_finalize_kernel adds in chunk order (bwd_head_chunks in common.cuh).
 // Roles (512 threads, at most 128 registers each): warp 0 TMA producer (+ TMEM owner);
 // three MMA issuers on different warps, each waiting only for its own operands:
 // warp 1 (one lane) dV_c and dK_c per 16-query quarter, warp 14 (whole warp, an
@@ -79,8 +79,8 @@ struct Params {
   const float* delta;  // [B][Hq][ns][Lvp]
   bf16* dk;
   bf16* dv;
-  float* dkv;   // head chunks > 1: fp32 partial sums [2][B][q_ns][Lv][Hkv][DH] (dV, dK)
-  int hchunks;  // query-head chunks per K/V head (bwd256_head_chunks)
+  float* dkv;   // head chunks > 1: fp32 partial sums [chunks][2][B][q_ns][Lv][Hkv][DH] (dV, dK)
+  int hchunks;  // query-head chunks per K/V head (bwd_head_chunks)
   SfaGeom g;
   float scale, scale_log2;
   int32_t* status;
@@ -127,7 +127,17 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
   const int T = grp * nq;
   const int Lqp = row_terms_pitch(G.Lq);
   if (nq <= 0) {  // no query sees this key tile: its half of the dK and dV rows is zero
-    if (HC > 1) return;  // the workspace rows stay zero; the finalize pass writes them
+    if (HC > 1) {  // this chunk's slice rows (its head-dim half) are zero
+      const size_t half = (size_t)G.B * G.q_ns * G.Lv * G.Hkv * DH;
+      for (int i = threadIdx.x; i < BK * (DHH / 4); i += NTHREADS) {
+        const int kr = n0 + i / (DHH / 4), c4 = i % (DHH / 4);
+        if (kr >= G.Lv) continue;
+        const long long wrow = ((((long long)b * G.q_ns + s) * G.Lv + kr) * G.Hkv + kvh) * DH + c * DHH + c4 * 4;
+        *reinterpret_cast<float4*>(P.dkv + (2 * hc) * half + wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
+        *reinterpret_cast<float4*>(P.dkv + (2 * hc + 1) * half + wrow) = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      return;
+    }
     for (int i = threadIdx.x; i < BK * (DHH / 8); i += NTHREADS) {
       const int kr = n0 + i / (DHH / 8), cc = i % (DHH / 8);
       if (kr >= G.Lv) continue;
@@ -398,8 +408,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
         }
       }
     }
-    // epilogue: this key row's half of dV, then of dK (scaled); with head chunks, added
-    // into the fp32 workspace instead (red.global.add, 16 bytes at a time)
+    // epilogue: this key row's half of dV, then of dK (scaled); with head chunks, into
+    // this chunk's fp32 workspace slice instead
     if (ok && __all_sync(0xffffffffu, mbar_wait(&sm.kv_done, 0, abort, P.status))) {
       tc_fence_after();
       const long long orow = (((long long)b * G.nL + (long long)kr * G.rs + sk) * G.Hkv + kvh) * DH + c * DHH;
@@ -416,11 +426,12 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
         tmem_ld_wait();
         if (HC > 1) {
           if (kr < G.Lv) {
-            float* wdst = P.dkv + which * half + wrow + (cc % (DHH / 32)) * 32;
+            float* wdst = P.dkv + (2 * hc + which) * half + wrow + (cc % (DHH / 32)) * 32;
 #pragma unroll
             for (int e = 0; e < 32; e += 4)
-              red_add_v4(wdst + e, __uint_as_float(ov[e]) * mul, __uint_as_float(ov[e + 1]) * mul,
-                         __uint_as_float(ov[e + 2]) * mul, __uint_as_float(ov[e + 3]) * mul);
+              *reinterpret_cast<float4*>(wdst + e) =
+                  make_float4(__uint_as_float(ov[e]) * mul, __uint_as_float(ov[e + 1]) * mul,
+                              __uint_as_float(ov[e + 2]) * mul, __uint_as_float(ov[e + 3]) * mul);
           }
         } else if (kr < G.Lv) {
 #pragma unroll
@@ -579,9 +590,10 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd256_kernel(const __grid_consta
     tmem_dealloc(tmem, 512);
   }
 }
-// Head chunks: dv / dk rows (bf16) from the fp32 partial sums, 8 columns per thread.
+// Head chunks: dv / dk rows (bf16) from the chunks' fp32 partial sums, added in chunk
+// order, 8 columns per thread.
 __global__ void __launch_bounds__(256) dkv_finalize_kernel(const float* __restrict__ dkv, bf16* __restrict__ dk,
-                                                           bf16* __restrict__ dv, SfaGeom g) {
+                                                           bf16* __restrict__ dv, SfaGeom g, int chunks) {
   const long long n8 = (long long)g.B * g.q_ns * g.Lv * g.Hkv * (DH / 8);
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n8) return;
@@ -596,8 +608,13 @@ __global__ void __launch_bounds__(256) dkv_finalize_kernel(const float* __restri
   const size_t half = (size_t)n8 * 8;
 #pragma unroll
   for (int which = 0; which < 2; ++which) {
-    const float4* src = reinterpret_cast<const float4*>(dkv + which * half + i * 8);
-    const float4 x = src[0], y = src[1];
+    float4 x = make_float4(0.f, 0.f, 0.f, 0.f), y = x;
+    for (int hc = 0; hc < chunks; ++hc) {
+      const float4* src = reinterpret_cast<const float4*>(dkv + (2 * hc + which) * half + i * 8);
+      const float4 a = src[0], e = src[1];
+      x.x += a.x; x.y += a.y; x.z += a.z; x.w += a.w;
+      y.x += e.x; y.y += e.y; y.z += e.z; y.w += e.w;
+    }
     uint4 w;
     w.x = cvt_bf16x2(x.x, x.y);
     w.y = cvt_bf16x2(x.z, x.w);
@@ -623,18 +640,14 @@ cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* 
   p.delta = delta_ws;
   p.dk = (bf16*)dk;
   p.dv = (bf16*)dv;
-  p.hchunks = bwd256_head_chunks(g);
+  p.hchunks = bwd_head_chunks(g, DH);
   p.dkv = dkv_ws;
   p.g = g;
   p.scale = scale;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.status = status;
-  const size_t nkv = bwd256_dkv_elems(g);
-  if (p.hchunks > 1) {
-    if (dkv_ws == nullptr) return cudaErrorInvalidValue;
-    cudaError_t e = cudaMemsetAsync(dkv_ws, 0, 2 * nkv * sizeof(float), st);
-    if (e != cudaSuccess) return e;
-  }
+  const size_t nkv = bwd_dkv_slice(g, DH);
+  if (p.hchunks > 1 && dkv_ws == nullptr) return cudaErrorInvalidValue;
   const int smem = kSmemBytes;
   auto kern = g.window > 0 ? bwd256_kernel<true> : bwd256_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -644,7 +657,7 @@ cudaError_t launch_sfa_bwd_main_tc256(const void* q, const void* k, const void* 
   e = cudaGetLastError();
   if (e != cudaSuccess || p.hchunks == 1) return e;
   const long long n8 = (long long)nkv / 8;
-  dkv_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dkv_ws, (bf16*)dk, (bf16*)dv, g);
+  dkv_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dkv_ws, (bf16*)dk, (bf16*)dv, g, p.hchunks);
   return cudaGetLastError();
 }
 

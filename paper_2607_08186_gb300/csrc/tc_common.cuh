@@ -216,12 +216,6 @@ HD_DEVINLINE uint64_t fmul2(uint64_t a, uint64_t b) {
   return d;
 }
 
-// *p += (a, b, c, d) as one 16-byte global reduction (p 16-byte aligned).
-HD_DEVINLINE void red_add_v4(float* p, float a, float b, float c, float d) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};\n" ::"l"(p), "f"(a), "f"(b), "f"(c), "f"(d)
-               : "memory");
-}
-
 // 32 TMEM lanes x 16 consecutive 32-bit columns (load) / 8 columns (store).
 HD_DEVINLINE void tmem_ld16(uint32_t taddr, uint32_t* r) {
   asm volatile(

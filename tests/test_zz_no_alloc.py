@@ -46,9 +46,9 @@ def test_rejects_sizes_beyond_the_fixed_workspace(lib):
 # (shape, mode, window); the later calls need less workspace than the first, so the
 # array still holds the first call's data past their own.
 # The first needs 63.5 MiB of the 64 MiB array (the split workspace's row terms sit at
-# its top end).
+# its top end; 16 K/V heads give a grid of 512 CTAs, so no head-chunk partial sums).
 CALLS = [
-    (AttnShape(1, 1000, 4, 32, 8, 128), WITHIN, 0),
+    (AttnShape(1, 1000, 4, 32, 16, 128), WITHIN, 0),
     (AttnShape(1, 200, 4, 8, 2, 128), WITHIN, 0),
     (AttnShape(1, 96, 2, 4, 4, 64), CROSS, 0),
     (AttnShape(2, 70, 2, 4, 2, 128), LOCAL, 50),
