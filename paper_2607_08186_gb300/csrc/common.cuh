@@ -58,7 +58,7 @@ __host__ __device__ inline int row_terms_pitch(int Lv) { return (Lv + kRowTermAl
 // Head chunks of the tensor-core backward.  Its grid is one CTA (two at head dim 256)
 // per 128-row key tile and (b, K/V head, stream); when that leaves SMs idle (short or
 // final-stream problems with few K/V heads), each CTA takes only a chunk of the group's
-// query heads, for about two CTAs per SM.  (With one to two CTAs per SM, as in the n = 1
+// query heads, for up to about four CTAs per SM.  (With one to two CTAs per SM, as in the n = 1
 // and the final-stream intra-stream layers with 8 K/V heads, the partial sums' extra
 // traffic cost more than the better balance gained: 3 % slower.)  Chunk hc writes its dK / dV partial sums (fp32,
 // dK already scaled) to its own slice of a workspace [chunks][2][B][q_ns][Lv][Hkv][Dh]
@@ -69,7 +69,7 @@ __host__ __device__ inline int bwd_head_chunks(const SfaGeom& g, int Dh) {
   const long long ctas = (long long)((g.Lv + 127) / 128) * (Dh == 256 ? 2 : 1) * g.Hkv * g.q_ns * g.B;
   const int grp = g.Hq / g.Hkv;
   if (ctas >= kSmCount || grp < 2) return 1;
-  long long want = (2 * kSmCount + ctas - 1) / ctas;
+  long long want = (4 * kSmCount + ctas - 1) / ctas;  // 2 or 6 per SM: 3.5 % / 1 % slower
   const int hs = (int)(want < grp ? want : grp);
   const int per = (grp + hs - 1) / hs;
   return (grp + per - 1) / per;
