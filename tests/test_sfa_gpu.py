@@ -82,6 +82,22 @@ def test_head_dim_256_many_key_tiles(mode, window):
     _full_case(AttnShape(1, 300, 4, 4, 2, 256), mode, seed=33, window=window)
 
 
+@pytest.mark.parametrize("mode,window", [(WITHIN, 0), (CROSS, 0), (LOCAL, 60)])
+@pytest.mark.parametrize("Dh", [64, 128, 256])
+def test_uneven_head_chunks(mode, window, Dh):
+    # 11 query heads per K/V head on a backward grid of 64 CTAs (128 at head dim 256):
+    # each group splits into head chunks of 2 (3) heads with a smaller last one, whose
+    # fp32 dK / dV partial sums the finalize pass adds in chunk order; against the
+    # oracle, and dK / dV bit-identical on a rerun (dQ's fp32 reduce-adds from many CTAs
+    # arrive in a run-dependent order: it agrees to rounding only)
+    s = AttnShape(4, 256, 4, 22, 2, Dh)
+    _full_case(s, mode, seed=41 + Dh, window=window)
+    q, k, v, do = inputs.attn_inputs(s, seed=41 + Dh)
+    runs = [gpu_fwd_bwd(q, k, v, do, s.n, mode, 0.0, window)[3:] for _ in range(2)]
+    for a, b in zip(*runs):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+
+
 @pytest.mark.parametrize("shape", [(1, 100, 1, 4, 2, 128), (1, 130, 4, 4, 1, 128), (2, 77, 3, 4, 2, 128),
                                    (1, 70, 8, 2, 2, 128)])
 def test_naive_within_schedule(shape):
