@@ -79,30 +79,6 @@ __host__ __device__ inline size_t bwd_dkv_slice(const SfaGeom& g, int Dh) {
   return bwd_head_chunks(g, Dh) > 1 ? (size_t)g.B * g.q_ns * g.Lv * g.Hkv * Dh : 0;
 }
 
-// Programmatic dependent launch.  A kernel launched with launch_pdl may start while the
-// previous kernel of its stream is still running: it lets its own dependents start as
-// early (pdl_trigger, at entry) and waits for its predecessors to complete, with their
-// memory visible, before its first global-memory access (pdl_wait).  Launched without
-// the attribute, both are no-ops.
-HD_DEVINLINE void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
-HD_DEVINLINE void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
-
-template <typename... KArgs, typename... Args>
-inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
-                              Args... args) {
-  cudaLaunchAttribute at[1];
-  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[0].val.programmaticStreamSerializationAllowed = 1;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = block;
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cfg.attrs = at;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, args...);
-}
-
 HD_DEVINLINE uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -13,8 +13,6 @@ __global__ void __launch_bounds__(256) expand_embed_kernel(const uint4* __restri
                                                            const int32_t* __restrict__ ids,
                                                            uint4* __restrict__ out, long long rows,
                                                            int n, int V, int D16, int32_t* status) {
-  pdl_trigger();
-  pdl_wait();
   const int lane = threadIdx.x & 31;
   const long long warp0 = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const long long nwarps = ((long long)gridDim.x * blockDim.x) >> 5;
@@ -47,8 +45,9 @@ cudaError_t launch_expand_embed(const void* tables, const int32_t* ids, void* ou
   const int threads = 256;
   long long blocks = (rows + (threads / 32) - 1) / (threads / 32);
   if (blocks > 152LL * 64) blocks = 152LL * 64;  // grid-stride beyond 64 waves of the 152 SMs
-  return launch_pdl(expand_embed_kernel, dim3((unsigned)blocks), dim3(threads), 0, stream, (const uint4*)tables, ids,
-                    (uint4*)out, rows, n, V, D / 8, status);
+  expand_embed_kernel<<<(unsigned)blocks, threads, 0, stream>>>(
+      (const uint4*)tables, ids, (uint4*)out, rows, n, V, D / 8, status);
+  return cudaGetLastError();
 }
 
 }  // namespace hdsfa

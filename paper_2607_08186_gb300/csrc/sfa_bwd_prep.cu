@@ -31,8 +31,6 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
                                                            float* __restrict__ lse2_t,
                                                            float* __restrict__ delta_t,
                                                            float* __restrict__ dq_acc, SfaGeom g) {
-  pdl_trigger();
-  pdl_wait();
   constexpr int LPR = DH / 8;      // lanes per row
   constexpr int RPG = 32 / LPR;    // rows per load instruction
   constexpr int RPW = 8;           // rows per warp
@@ -100,15 +98,11 @@ __global__ void __launch_bounds__(256) sfa_bwd_prep_kernel(const bf16* __restric
 
 // The fp32 dQ accumulator alone, zeroed with 16-byte stores (grid-stride).
 __global__ void __launch_bounds__(256) sfa_bwd_clear_kernel(float4* __restrict__ acc, long long n4) {
-  pdl_trigger();
-  pdl_wait();
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (long long)gridDim.x * blockDim.x)
     acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 __global__ void sfa_bwd_pad_kernel(float* __restrict__ lse2_t, float* __restrict__ delta_t, SfaGeom g) {
-  pdl_trigger();
-  pdl_wait();
   const int Lvp = row_terms_pitch(g.Lv), pad = Lvp - g.Lv;
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= (long long)g.B * g.Hq * g.ns * pad) return;
@@ -120,8 +114,6 @@ __global__ void sfa_bwd_pad_kernel(float* __restrict__ lse2_t, float* __restrict
 __global__ void __launch_bounds__(256) sfa_bwd_finalize_kernel(const float* __restrict__ dq_acc,
                                                                bf16* __restrict__ dq, long long n8,
                                                                float scale) {
-  pdl_trigger();
-  pdl_wait();
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n8) return;
   const float4 a = reinterpret_cast<const float4*>(dq_acc)[2 * i];
@@ -140,28 +132,29 @@ cudaError_t launch_sfa_bwd_prep(const void* o, const void* dout, const float* ls
   const long long warps = (long long)g.B * g.ns * ((g.Lv + 7) / 8) * g.Hq;  // 8 rows of one problem each
   const unsigned blocks = (unsigned)((warps * 32 + 255) / 256);
   const bf16 *ob = (const bf16*)o, *db = (const bf16*)dout;
-  cudaError_t e;
   if (Dh == 256) {
     if (zero)
-      e = launch_pdl(sfa_bwd_prep_kernel<256, true>, dim3(blocks), dim3(256), 0, st, ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+      sfa_bwd_prep_kernel<256, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
     else
-      e = launch_pdl(sfa_bwd_prep_kernel<256, false>, dim3(blocks), dim3(256), 0, st, ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+      sfa_bwd_prep_kernel<256, false><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
   } else if (Dh == 64) {
     if (zero)
-      e = launch_pdl(sfa_bwd_prep_kernel<64, true>, dim3(blocks), dim3(256), 0, st, ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+      sfa_bwd_prep_kernel<64, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
     else
-      e = launch_pdl(sfa_bwd_prep_kernel<64, false>, dim3(blocks), dim3(256), 0, st, ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+      sfa_bwd_prep_kernel<64, false><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
   } else {
     if (zero)
-      e = launch_pdl(sfa_bwd_prep_kernel<128, true>, dim3(blocks), dim3(256), 0, st, ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+      sfa_bwd_prep_kernel<128, true><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
     else
-      e = launch_pdl(sfa_bwd_prep_kernel<128, false>, dim3(blocks), dim3(256), 0, st, ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
+      sfa_bwd_prep_kernel<128, false><<<blocks, 256, 0, st>>>(ob, db, lse, lse2_ws, delta_ws, dq_ws, g);
   }
+  cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int pad = row_terms_pitch(g.Lv) - g.Lv;
   if (pad > 0) {
     const long long n = (long long)g.B * g.Hq * g.ns * pad;
-    e = launch_pdl(sfa_bwd_pad_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, st, lse2_ws, delta_ws, g);
+    sfa_bwd_pad_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(lse2_ws, delta_ws, g);
+    e = cudaGetLastError();
   }
   return e;
 }
@@ -170,15 +163,15 @@ cudaError_t launch_sfa_bwd_clear(float* dq_ws, const SfaGeom& g, int Dh, cudaStr
   const long long n4 = (long long)g.B * g.nL * g.Hq * Dh / 4;
   long long blocks = (n4 + 255) / 256;
   if (blocks > 152LL * 16) blocks = 152LL * 16;
-  return launch_pdl(sfa_bwd_clear_kernel, dim3((unsigned)blocks), dim3(256), 0, st, reinterpret_cast<float4*>(dq_ws),
-                    n4);
+  sfa_bwd_clear_kernel<<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<float4*>(dq_ws), n4);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_sfa_bwd_finalize(void* dq, const float* dq_ws, const SfaGeom& g, int Dh,
                                     float scale, cudaStream_t st) {
   const long long n8 = (long long)g.B * g.nL * g.Hq * Dh / 8;
-  return launch_pdl(sfa_bwd_finalize_kernel, dim3((unsigned)((n8 + 255) / 256)), dim3(256), 0, st, dq_ws, (bf16*)dq,
-                    n8, scale);
+  sfa_bwd_finalize_kernel<<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(dq_ws, (bf16*)dq, n8, scale);
+  return cudaGetLastError();
 }
 
 }  // namespace hdsfa

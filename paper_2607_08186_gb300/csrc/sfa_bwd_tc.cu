@@ -110,7 +110,6 @@ struct Params {
 // of them instead of 64; S^T, dP^T and the pre-fills are as at 128.
 template <int DH, bool WIN>
 __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant__ Params P) {
-  pdl_trigger();  // launched with launch_pdl: waits for its predecessor below
   static_assert(DH == 64 || DH == 128, "head dim 64 or 128");
   extern __shared__ uint8_t smem_raw[];
   {
@@ -118,7 +117,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     asm("mov.u32 %0, %%dynamic_smem_size;\n" : "=r"(dyn));
     const uintptr_t base = reinterpret_cast<uintptr_t>(smem_raw);
     if (((base + 1023) & ~uintptr_t(1023)) - base + sizeof(Smem<DH>) > dyn) {  // uniform: nothing touched yet
-      pdl_wait();
       if (threadIdx.x == 0) set_status(P.status, HD_DEVBIT_TIMEOUT);
       return;
     }
@@ -150,7 +148,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
   const int T = grp * nq;
   const int Lqp = row_terms_pitch(G.Lq);
   if (nq <= 0) {  // no query sees this key tile: its dK and dV rows are zero
-    pdl_wait();
     if (HC > 1) {  // this chunk's slice rows are zero
       const size_t half = (size_t)G.B * G.q_ns * G.Lv * G.Hkv * DH;
       for (int i = threadIdx.x; i < BK * (DH / 4); i += NTHREADS) {
@@ -202,7 +199,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
     tmem_alloc(&sm.tmem_base, 512);
     tmem_relinquish();
   }
-  pdl_wait();  // the set-up above overlaps the previous kernel's tail; memory after this
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -678,8 +674,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) bwd_kernel(const __grid_constant_
 template <int DH>
 __global__ void __launch_bounds__(256) dkv_finalize_kernel(const float* __restrict__ dkv, bf16* __restrict__ dk,
                                                            bf16* __restrict__ dv, SfaGeom g, int chunks) {
-  pdl_trigger();
-  pdl_wait();
   const long long n8 = (long long)g.B * g.q_ns * g.Lv * g.Hkv * (DH / 8);
   const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n8) return;
@@ -721,11 +715,12 @@ static cudaError_t bwd_tc_impl(tcbwd::Params& p, const SfaGeom& g, cudaStream_t 
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const unsigned grid = (unsigned)((g.Lv + BK - 1) / BK) * (unsigned)(p.hchunks * g.Hkv * g.q_ns * g.B);
-  e = launch_pdl(kern, dim3(grid), dim3(NTHREADS), (size_t)smem, st, p);
+  kern<<<grid, NTHREADS, smem, st>>>(p);
+  e = cudaGetLastError();
   if (e != cudaSuccess || p.hchunks == 1) return e;
   const long long n8 = (long long)nkv / 8;
-  return launch_pdl(dkv_finalize_kernel<DH>, dim3((unsigned)((n8 + 255) / 256)), dim3(256), 0, st, p.dkv, p.dk, p.dv,
-                    g, p.hchunks);
+  dkv_finalize_kernel<DH><<<(unsigned)((n8 + 255) / 256), 256, 0, st>>>(p.dkv, p.dk, p.dv, g, p.hchunks);
+  return cudaGetLastError();
 }
 
 // Dh: 64 or 128.

@@ -81,7 +81,6 @@ HD_DEVINLINE void tile_range(const SfaGeom& G, int m0, int& lo, int& hi) {
 // modes' softmax carries none of that code.
 template <int DH, bool NAIVE>
 __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant__ Params P) {
-  pdl_trigger();  // launched with launch_pdl: waits for its predecessor below
   extern __shared__ uint8_t smem_raw[];
   Smem<DH>& sm = *reinterpret_cast<Smem<DH>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const SfaGeom& G = P.g;
@@ -135,7 +134,6 @@ __global__ void __launch_bounds__(NTHREADS, 1) fwd_kernel(const __grid_constant_
     tmem_alloc(&sm.tmem_base, 512);
     tmem_relinquish();
   }
-  pdl_wait();  // the set-up above overlaps the previous kernel's tail; memory after this
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -396,7 +394,8 @@ static cudaError_t tc_fwd_impl(tcfwd::Params& p, cudaStream_t st) {
   const int rows_per_cta = p.head_pairs ? tcfwd::BM : tcfwd::NG * tcfwd::BM;
   const int nh = p.head_pairs ? p.g.Hq / tcfwd::NG : p.g.Hq;
   const unsigned grid = (unsigned)((p.g.Lq + rows_per_cta - 1) / rows_per_cta) * (unsigned)(nh * p.g.q_ns * p.g.B);
-  return launch_pdl(tcfwd::fwd_kernel<DH, NAIVE>, dim3(grid), dim3(tcfwd::NTHREADS), (size_t)smem, st, p);
+  tcfwd::fwd_kernel<DH, NAIVE><<<grid, tcfwd::NTHREADS, smem, st>>>(p);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_sfa_fwd_tc(const void* q, const void* k, const void* v, void* o, float* lse,
