@@ -217,6 +217,23 @@ def test_qwen3_8b_class_layer(mode):
 
 
 @pytest.mark.parametrize("mode", [WITHIN, CROSS])
+def test_qwen3_8b_class_layer_one_group_complete(mode):
+    # the benchmark layer (B=1, L=4096, n=4, Hq=32, Hkv=8, Dh=128) with one K/V head group
+    # checked whole: O and LSE of its 4 query heads at every position, dQ of those heads
+    # and dK, dV of its K/V head at every position, against the oracle over the group
+    s = inputs.SHAPES["qwen3_8b_n4"]
+    q, k, v, do = inputs.attn_inputs(s, seed=1)
+    o, lse, dq, dk, dv = gpu_fwd_bwd(q, k, v, do, s.n, mode)
+    grp, g = s.Hq // s.Hkv, 5
+    hs = slice(g * grp, (g + 1) * grp)
+    qg, kg, vg, dog = group_slices(q, k, v, do, g, grp)
+    o_r, l_r = oracle.sfa_fwd(qg, kg, vg, s.n, mode)
+    assert_fwd_close(o[:, :, hs], lse[:, hs], o_r, l_r)
+    dq_r, dk_r, dv_r = oracle.sfa_bwd(qg, kg, vg, dog, s.n, mode)
+    assert_grads_close([("dq", dq[:, :, hs], dq_r), ("dk", dk[:, :, g:g + 1], dk_r), ("dv", dv[:, :, g:g + 1], dv_r)])
+
+
+@pytest.mark.parametrize("mode", [WITHIN, CROSS])
 def test_large_moe_class_layer(mode):
     # B=1, L=8192, n=4 (32768 positions), Hq=64, Hkv=8, Dh=128
     _sampled_parity(inputs.SHAPES["moe_large_n4"], mode, seed=21, n_rows=96, n_kv=24, repeat=True)
